@@ -1,0 +1,205 @@
+/*
+ * qx_oracle.c -- TEST INFRASTRUCTURE ONLY.
+ *
+ * A plain, slow, obviously-correct CPU statement of what the exact integer
+ * matrix-multiplication substrate computes.  Only tests/, the smoke check in
+ * __graft_entry__.py and the CPU-baseline leg of bench.py may load it.  The
+ * CUDA library never links, includes or calls anything here, and nothing here
+ * knows about limbs, tiles, chunks or any other device-side technique.
+ *
+ * What is computed (all from the paper's Methodology paragraph, Table 1 and
+ * Table 2):
+ *   - INT16-input / INT32-accumulation GEMM and INT32-operand GEMM
+ *     (Abstract; Methodology; Table 1):  C[i][j] = sum_k A[i][k] * B[k][j].
+ *     Operands arrive as int32 (int16 values widen losslessly); the sum is
+ *     carried in int64, so it is the exact integer result.  The routine also
+ *     reports the largest |partial sum| seen, in the order k = 0, 1, ..., so a
+ *     caller can check the int32 accumulation contract (Methodology: operand-
+ *     range contracts bound what the accumulation must hold).
+ *   - GEMM-backed Conv2D (Methodology: "convolution ... through lowering";
+ *     Table 2).  The oracle is the direct convolution itself, not a lowering:
+ *     y[n][o][p][q] = sum_c sum_r sum_s x[n][c][p*st-pad+r][q*st-pad+s]
+ *                                       * w[o][c][r][s],
+ *     zero outside the image; NCHW input, KCRS weights, cross-correlation (no
+ *     kernel flip), no bias.
+ *   - Single-head attention core O = (Q K^T) V, no softmax, no scale
+ *     (Methodology; Table 2), computed as written: first S = Q K^T, then
+ *     O = S V.
+ *   - FP64 versions of the three operators for the FP32 variants of Table 2.
+ *     The tolerance reference sum_k |a_k||b_k| is the same routine applied to
+ *     element-wise absolute values (the Python wrapper does that).
+ *
+ * Loop order: the GEMM runs i-k-j with a per-row int64 accumulator row, which
+ * visits the k terms of every C[i][j] in increasing k exactly like the i-j-k
+ * definition (integer addition is exact, so only the partial-sum trace could
+ * differ, and it does not).  Rows are independent; OpenMP splits them.
+ */
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+static inline int64_t abs64(int64_t v) { return v < 0 ? -v : v; }
+
+int qxo_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/* C = A * B.  A is M x K (row pitch lda), B is K x N (row pitch ldb), C is
+ * M x N (row pitch ldc), all row-major.  max_abs_partial (may be NULL) gets
+ * max over i, j, k of |sum_{t<=k} A[i][t] B[t][j]|. */
+void qxo_gemm_i64(int64_t M, int64_t N, int64_t K,
+                  const int32_t *A, int64_t lda,
+                  const int32_t *B, int64_t ldb,
+                  int64_t *C, int64_t ldc, int64_t *max_abs_partial)
+{
+    int64_t worst = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(max : worst)
+    for (int64_t i = 0; i < M; ++i) {
+        int64_t *row = C + i * ldc;
+        int64_t row_worst = 0;
+        for (int64_t j = 0; j < N; ++j) row[j] = 0;
+        for (int64_t k = 0; k < K; ++k) {
+            const int64_t a = A[i * lda + k];
+            const int32_t *b = B + k * ldb;
+            for (int64_t j = 0; j < N; ++j) {
+                row[j] += a * (int64_t)b[j];
+                int64_t m = abs64(row[j]);
+                row_worst = m > row_worst ? m : row_worst;
+            }
+        }
+        worst = row_worst > worst ? row_worst : worst;
+    }
+    if (max_abs_partial) *max_abs_partial = worst;
+}
+
+/* Direct convolution, NCHW x (n, c, h, w), KCRS weights (k, c, r, s),
+ * y (n, k, P, Q) with P = (h + 2 pad - r) / stride + 1, Q likewise. */
+void qxo_conv2d_i64(int64_t n, int64_t c, int64_t h, int64_t w,
+                    int64_t k, int64_t r, int64_t s,
+                    int64_t stride, int64_t pad,
+                    const int32_t *x, const int32_t *wt, int64_t *y)
+{
+    const int64_t P = (h + 2 * pad - r) / stride + 1;
+    const int64_t Q = (w + 2 * pad - s) / stride + 1;
+#pragma omp parallel for collapse(2) schedule(dynamic, 1)
+    for (int64_t in = 0; in < n; ++in)
+        for (int64_t o = 0; o < k; ++o)
+            for (int64_t p = 0; p < P; ++p)
+                for (int64_t q = 0; q < Q; ++q) {
+                    int64_t acc = 0;
+                    for (int64_t ic = 0; ic < c; ++ic)
+                        for (int64_t fr = 0; fr < r; ++fr)
+                            for (int64_t fs = 0; fs < s; ++fs) {
+                                const int64_t ih = p * stride - pad + fr;
+                                const int64_t iw = q * stride - pad + fs;
+                                if (ih < 0 || ih >= h || iw < 0 || iw >= w) continue;
+                                acc += (int64_t)x[((in * c + ic) * h + ih) * w + iw] *
+                                       (int64_t)wt[((o * c + ic) * r + fr) * s + fs];
+                            }
+                    y[((in * k + o) * P + p) * Q + q] = acc;
+                }
+}
+
+/* Attention core as written: S = Q K^T (L x L), then O = S V (L x d).
+ * Q, K, V are L x d row-major.  S may be NULL (then a scratch copy is used).
+ * max_abs_s (may be NULL) gets max |S[i][j]|. */
+void qxo_attn_i64(int64_t L, int64_t d,
+                  const int32_t *Qm, const int32_t *Km, const int32_t *Vm,
+                  int64_t *S, int64_t *O, int64_t *max_abs_s)
+{
+    int64_t *Sb = S ? S : (int64_t *)malloc((size_t)(L * L) * sizeof(int64_t));
+    int64_t worst = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(max : worst)
+    for (int64_t i = 0; i < L; ++i)
+        for (int64_t j = 0; j < L; ++j) {
+            int64_t acc = 0;
+            for (int64_t m = 0; m < d; ++m)
+                acc += (int64_t)Qm[i * d + m] * (int64_t)Km[j * d + m];
+            Sb[i * L + j] = acc;
+            int64_t a = abs64(acc);
+            worst = a > worst ? a : worst;
+        }
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t i = 0; i < L; ++i)
+        for (int64_t cc = 0; cc < d; ++cc) {
+            int64_t acc = 0;
+            for (int64_t j = 0; j < L; ++j)
+                acc += Sb[i * L + j] * (int64_t)Vm[j * d + cc];
+            O[i * d + cc] = acc;
+        }
+    if (max_abs_s) *max_abs_s = worst;
+    if (!S) free(Sb);
+}
+
+/* ---- FP64 versions (same definitions, double arithmetic) ---- */
+
+void qxo_gemm_f64(int64_t M, int64_t N, int64_t K,
+                  const double *A, int64_t lda, const double *B, int64_t ldb,
+                  double *C, int64_t ldc)
+{
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t i = 0; i < M; ++i) {
+        double *row = C + i * ldc;
+        for (int64_t j = 0; j < N; ++j) row[j] = 0.0;
+        for (int64_t k = 0; k < K; ++k) {
+            const double a = A[i * lda + k];
+            const double *b = B + k * ldb;
+            for (int64_t j = 0; j < N; ++j) row[j] += a * b[j];
+        }
+    }
+}
+
+void qxo_conv2d_f64(int64_t n, int64_t c, int64_t h, int64_t w,
+                    int64_t k, int64_t r, int64_t s,
+                    int64_t stride, int64_t pad,
+                    const double *x, const double *wt, double *y)
+{
+    const int64_t P = (h + 2 * pad - r) / stride + 1;
+    const int64_t Q = (w + 2 * pad - s) / stride + 1;
+#pragma omp parallel for collapse(2) schedule(dynamic, 1)
+    for (int64_t in = 0; in < n; ++in)
+        for (int64_t o = 0; o < k; ++o)
+            for (int64_t p = 0; p < P; ++p)
+                for (int64_t q = 0; q < Q; ++q) {
+                    double acc = 0.0;
+                    for (int64_t ic = 0; ic < c; ++ic)
+                        for (int64_t fr = 0; fr < r; ++fr)
+                            for (int64_t fs = 0; fs < s; ++fs) {
+                                const int64_t ih = p * stride - pad + fr;
+                                const int64_t iw = q * stride - pad + fs;
+                                if (ih < 0 || ih >= h || iw < 0 || iw >= w) continue;
+                                acc += x[((in * c + ic) * h + ih) * w + iw] *
+                                       wt[((o * c + ic) * r + fr) * s + fs];
+                            }
+                    y[((in * k + o) * P + p) * Q + q] = acc;
+                }
+}
+
+void qxo_attn_f64(int64_t L, int64_t d,
+                  const double *Qm, const double *Km, const double *Vm,
+                  double *S, double *O)
+{
+    double *Sb = S ? S : (double *)malloc((size_t)(L * L) * sizeof(double));
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t i = 0; i < L; ++i)
+        for (int64_t j = 0; j < L; ++j) {
+            double acc = 0.0;
+            for (int64_t m = 0; m < d; ++m) acc += Qm[i * d + m] * Km[j * d + m];
+            Sb[i * L + j] = acc;
+        }
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t i = 0; i < L; ++i)
+        for (int64_t cc = 0; cc < d; ++cc) {
+            double acc = 0.0;
+            for (int64_t j = 0; j < L; ++j) acc += Sb[i * L + j] * Vm[j * d + cc];
+            O[i * d + cc] = acc;
+        }
+    if (!S) free(Sb);
+}

@@ -1,0 +1,245 @@
+"""Pins for the CPU oracle: it is checked against things other than itself.
+
+Each test ties the oracle to a hand-derived example, a closed form, an
+invariant, or an independent library routine (numpy int64 / float64 matmul,
+torch float64 conv2d), so that a dropped term, a wrong sign or index, a wrong
+padding rule or a transposed operand in the oracle fails at least one of them.
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_09905_gb300 import inputs
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "hand_examples.json")
+
+
+@pytest.fixture(scope="module")
+def golden():
+    with open(GOLDEN) as f:
+        return json.load(f)
+
+
+# ------------------------------------------------------------------ GEMM pins
+def test_gemm_hand_example(golden):
+    g = golden["gemm_2x3x2"]
+    C, _ = oracle.gemm(np.array(g["A"]), np.array(g["B"]))
+    assert C.tolist() == g["C"]
+
+
+def test_gemm_identity_and_permutation():
+    rng = np.random.default_rng(1)
+    A = rng.integers(-1023, 1024, size=(7, 5))
+    B = rng.integers(-1023, 1024, size=(5, 9))
+    assert (oracle.gemm(np.eye(7, dtype=np.int64), A)[0] == A).all()
+    assert (oracle.gemm(A, np.eye(5, dtype=np.int64))[0] == A).all()
+    perm = rng.permutation(5)
+    P = np.eye(5, dtype=np.int64)[perm]          # row-permutation matrix
+    assert (oracle.gemm(P, B)[0] == B[perm]).all()
+    Pc = np.eye(9, dtype=np.int64)[:, rng.permutation(9)]
+    assert (oracle.gemm(B, Pc)[0] == B @ Pc).all()
+
+
+@pytest.mark.parametrize("M,N,K,a,b", [(3, 4, 5, 2, -3), (1, 1, 1, -1023, 1023),
+                                       (8, 3, 256, 1023, 1023), (4, 4, 2048, -1023, 1023)])
+def test_gemm_constant_closed_form(M, N, K, a, b):
+    C, worst = oracle.gemm(np.full((M, K), a), np.full((K, N), b))
+    assert (C == K * a * b).all()
+    assert worst == K * abs(a * b)
+
+
+def test_gemm_rank_one_closed_form():
+    u = np.arange(-3, 4).reshape(7, 1)
+    v = np.array([[2, -1, 5, 0]])
+    w = np.array([[1, 2], [3, 4], [5, 6], [7, 8]])
+    C, _ = oracle.gemm(u @ v, w)          # (u v^T) w = u (v^T w)
+    assert (C == u * (v @ w)).all()
+
+
+@pytest.mark.parametrize("shape", [(1, 1, 1), (2, 3, 4), (17, 33, 65), (64, 96, 130)])
+def test_gemm_matches_numpy_int64(shape):
+    M, N, K = shape
+    A, B = inputs.gemm_case(M, N, K, -1023, 1023, seed=M + N + K)
+    C, _ = oracle.gemm(A, B)
+    ref = A.numpy().astype(np.int64) @ B.numpy().astype(np.int64)
+    assert (C == ref).all()
+
+
+def test_gemm_brute_force_tiny():
+    # every 2x2 A with entries in {-1, 0, 1} against a fixed asymmetric B set
+    vals = np.array([-1, 0, 1])
+    As = np.array(np.meshgrid(vals, vals, vals, vals)).T.reshape(-1, 2, 2)
+    Bs = As[::7]
+    for A in As:
+        for B in Bs:
+            assert (oracle.gemm(A, B)[0] == A @ B).all()
+
+
+def test_gemm_int32_operands_and_partial_trace():
+    # operands beyond int16 (smul24-sized) pass through unchanged
+    A = np.array([[2**22, -(2**22) + 1]], dtype=np.int32)
+    B = np.array([[3], [3]], dtype=np.int32)
+    C, worst = oracle.gemm(A, B)
+    assert C[0, 0] == 3
+    assert worst == 3 * 2**22                   # first partial sum is the largest
+    # partial sums that leave int32 are reported even when the total does not
+    A = np.array([[32767] * 3 + [-32767] * 3])
+    B = np.full((6, 1), 32767)
+    C, worst = oracle.gemm(A, B)
+    assert C[0, 0] == 0 and worst == 3 * 32767 * 32767 > 2**31 - 1
+
+
+def test_gemm_freivalds_consistency():
+    A, B = inputs.gemm_case(96, 80, 300, -1023, 1023, seed=5)
+    C, _ = oracle.gemm(A, B)
+    A = A.numpy().astype(np.int64)
+    B = B.numpy().astype(np.int64)
+    rng = np.random.default_rng(0)
+    for _ in range(4):
+        x = rng.choice([-1, 1], size=(80, 1))
+        assert (A @ (B @ x) == C @ x).all()
+
+
+def test_gemm_empty():
+    C, worst = oracle.gemm(np.zeros((0, 5), np.int16), np.zeros((5, 3), np.int16))
+    assert C.shape == (0, 3) and worst == 0
+    C, _ = oracle.gemm(np.zeros((2, 0), np.int16), np.zeros((0, 3), np.int16))
+    assert (C == 0).all() and C.shape == (2, 3)
+
+
+# ------------------------------------------------------------------ Conv pins
+@pytest.mark.parametrize("key", ["conv_3x3_k2_pad1", "conv_3x3_k2_pad0",
+                                 "conv_3x3_k2_pad1_stride2"])
+def test_conv_hand_examples(golden, key):
+    g = golden[key]
+    y = oracle.conv2d(np.array(g["x"]), np.array(g["w"]), g["stride"], g["pad"])
+    assert y.tolist() == g["y"]
+
+
+def test_conv_delta_kernels():
+    rng = np.random.default_rng(2)
+    x = rng.integers(-255, 256, size=(2, 3, 6, 5))
+    w = np.zeros((3, 3, 3, 3), dtype=np.int64)
+    for c in range(3):
+        w[c, c, 1, 1] = 1                           # centre tap: identity
+    assert (oracle.conv2d(x, w, 1, 1) == x).all()
+    w = np.zeros((3, 3, 3, 3), dtype=np.int64)
+    for c in range(3):
+        w[c, (c + 1) % 3, 0, 0] = 1                 # top-left tap, channel rotation
+    y = oracle.conv2d(x, w, 1, 1)
+    ref = np.zeros_like(x)
+    ref[:, :, 1:, 1:] = np.roll(x, -1, axis=1)[:, :, :-1, :-1]
+    assert (y == ref).all()
+
+
+def test_conv_all_ones_closed_form():
+    C = 5
+    y = oracle.conv2d(np.ones((1, C, 6, 7), np.int32), np.ones((2, C, 3, 3), np.int32), 1, 1)
+    exp = np.full((6, 7), 9 * C)
+    exp[0, :] = exp[-1, :] = 6 * C
+    exp[:, 0] = exp[:, -1] = 6 * C
+    exp[0, 0] = exp[0, -1] = exp[-1, 0] = exp[-1, -1] = 4 * C
+    assert (y[0, 0] == exp).all() and (y[0, 1] == exp).all()
+
+
+@pytest.mark.parametrize("stride,pad,shape", [(1, 1, (2, 4, 9, 7, 6, 3, 3)),
+                                              (2, 1, (1, 3, 8, 8, 5, 3, 3)),
+                                              (1, 0, (1, 2, 5, 6, 3, 1, 2)),
+                                              (2, 2, (1, 2, 7, 5, 2, 5, 3))])
+def test_conv_matches_torch_float64(stride, pad, shape):
+    n, c, h, w, k, r, s = shape
+    x, wt = inputs.conv_case(n, c, h, w, k, r, s, -255, 255, seed=sum(shape))
+    y = oracle.conv2d(x, wt, stride, pad)
+    ref = torch.nn.functional.conv2d(x.double(), wt.double(), stride=stride, padding=pad)
+    assert (y == ref.numpy().astype(np.int64)).all()
+
+
+def test_conv_matches_explicit_lowering():
+    # an independent route: materialised patch matrix times a numpy matmul
+    x, wt = inputs.conv_case(2, 4, 7, 6, 5, 3, 3, -255, 255, seed=3)
+    x = x.numpy().astype(np.int64)
+    wt = wt.numpy().astype(np.int64)
+    xp = np.pad(x, ((0, 0), (0, 0), (1, 1), (1, 1)))
+    cols = np.stack([xp[:, :, r:r + 7, s:s + 6] for r in range(3) for s in range(3)], axis=2)
+    cols = cols.reshape(2, 4 * 9, 7 * 6)                  # (n, c*r*s, P*Q), c-major
+    y_ref = np.einsum("ok,nkp->nop", wt.reshape(5, 36), cols).reshape(2, 5, 7, 6)
+    assert (oracle.conv2d(x, wt, 1, 1) == y_ref).all()
+
+
+# ------------------------------------------------------------- Attention pins
+def test_attn_hand_example(golden):
+    g = golden["attn_2x2"]
+    O, S, worst = oracle.attn(np.array(g["Q"]), np.array(g["K"]), np.array(g["V"]))
+    assert S.tolist() == g["S"] and O.tolist() == g["O"] and worst == 6
+
+
+def test_attn_identity_and_reassociation():
+    rng = np.random.default_rng(4)
+    V = rng.integers(-7, 8, size=(16, 16))
+    I = np.eye(16, dtype=np.int64)
+    O, S, _ = oracle.attn(I, I, V)
+    assert (S == I).all() and (O == V).all()
+    Q, K, V = (rng.integers(-7, 8, size=(40, 8)) for _ in range(3))
+    O, _, _ = oracle.attn(Q, K, V)
+    assert (O == Q @ (K.T @ V)).all()           # (Q K^T) V = Q (K^T V), exact
+
+
+def test_attn_extremes_and_numpy():
+    L, d = 24, 64
+    Q = np.full((L, d), 7)
+    K = np.full((L, d), -7)
+    V = np.full((L, d), 7)
+    O, S, worst = oracle.attn(Q, K, V)
+    assert worst == 3136 and (S == -3136).all() and (O == -3136 * 7 * L).all()
+    Q, K, V = inputs.attn_case(33, 10, -7, 7, seed=9)
+    O, S, _ = oracle.attn(Q, K, V)
+    q, k, v = (t.numpy().astype(np.int64) for t in (Q, K, V))
+    assert (S == q @ k.T).all() and (O == (q @ k.T) @ v).all()
+
+
+# ----------------------------------------------------------------- FP64 pins
+def test_f64_integer_valued_inputs_are_exact():
+    A, B = inputs.gemm_case(20, 30, 40, -1023, 1023, seed=11)
+    assert (oracle.gemm_f64(A.double(), B.double()) == oracle.gemm(A, B)[0]).all()
+    x, w = inputs.conv_case(1, 3, 6, 6, 4, 3, 3, -255, 255, seed=12)
+    assert (oracle.conv2d_f64(x.double(), w.double(), 1, 1) == oracle.conv2d(x, w, 1, 1)).all()
+    Q, K, V = inputs.attn_case(12, 8, -7, 7, seed=13)
+    assert (oracle.attn_f64(Q.double(), K.double(), V.double())[0] == oracle.attn(Q, K, V)[0]).all()
+
+
+def test_f64_matches_library_routines():
+    g = torch.Generator().manual_seed(14)
+    A = torch.randn(33, 47, generator=g, dtype=torch.float64)
+    B = torch.randn(47, 29, generator=g, dtype=torch.float64)
+    np.testing.assert_allclose(oracle.gemm_f64(A, B), (A @ B).numpy(), rtol=0, atol=1e-12)
+    x = torch.randn(2, 3, 9, 8, generator=g, dtype=torch.float64)
+    w = torch.randn(4, 3, 3, 3, generator=g, dtype=torch.float64)
+    ref = torch.nn.functional.conv2d(x, w, padding=1).numpy()
+    np.testing.assert_allclose(oracle.conv2d_f64(x, w, 1, 1), ref, rtol=0, atol=1e-12)
+    Q, K, V = (torch.randn(20, 6, generator=g, dtype=torch.float64) for _ in range(3))
+    np.testing.assert_allclose(oracle.attn_f64(Q, K, V)[0], ((Q @ K.T) @ V).numpy(),
+                               rtol=0, atol=1e-11)
+
+
+def test_absref_definition():
+    A = np.array([[1.0, -2.0], [-3.0, 4.0]])
+    B = np.array([[-5.0], [6.0]])
+    assert oracle.gemm_absref(A, B).tolist() == [[17.0], [39.0]]
+
+
+def test_fp32_as_written_meets_tolerance_reading():
+    # The FP32 tolerance reading max|err| <= 1e-5 * sum|a||b| must admit a
+    # plain FP32 evaluation of each operator (it is the bar the GPU path
+    # is held to).
+    x, w = inputs.conv_case_f32(2, 64, 10, 10, 8, 3, 3, seed=15)
+    ref = oracle.conv2d_f64(x, w, 1, 1)
+    got = torch.nn.functional.conv2d(x, w, padding=1).numpy()
+    assert (np.abs(got - ref) <= 1e-5 * oracle.conv2d_absref(x, w, 1, 1)).all()
+    Q, K, V = inputs.attn_case_f32(128, 64, seed=16)
+    ref, _ = oracle.attn_f64(Q, K, V)
+    got = ((Q @ K.T) @ V).numpy()
+    assert (np.abs(got - ref) <= 1e-5 * oracle.attn_absref(Q, K, V)).all()
