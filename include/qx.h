@@ -1,0 +1,167 @@
+/*
+ * qx.h -- C ABI of the exact integer GEMM substrate (GB300, sm_103a).
+ *
+ * The library implements the paper's data-parallel hot path: one tiled
+ * integer matrix-multiplication substrate (Abstract; Methodology paragraph)
+ * that serves
+ *   - packed INT16-input / INT32-accumulation GEMM      (Table 1, right half)
+ *   - INT32-operand GEMM under an operand-range contract (Table 1, left half;
+ *     Methodology: integer kernels obey the smul24 operand-range contract)
+ *   - GEMM-backed Conv2D through lowering               (Methodology; Table 2)
+ *   - the single-head attention core O = (Q K^T) V      (Methodology; Table 2)
+ * behind a persistent executor: a plan fixes shapes, dtypes and the operand-
+ * range contract, allocates device buffers once and caches every launch
+ * argument, so repeated execution does no setup work (Methodology: persistent
+ * executors allocate once and cache uniforms and dispatch metadata).
+ *
+ * Conventions for every call below
+ *   - Device pointers are CUDA device addresses on the plan's device; host
+ *     pointers are named as such.  The caller owns every operand and output
+ *     buffer; the plan owns its workspace.
+ *   - Execution calls are asynchronous on `stream` (a cudaStream_t; NULL is
+ *     the legacy default stream).  Argument errors are detected on the host
+ *     and returned before anything is launched.
+ *   - One plan must not run concurrently on two streams: calls share the
+ *     plan's workspace.  Distinct plans are independent.
+ *   - Operand base pointers must be 16-byte aligned.  Leading dimensions are
+ *     in elements and at least the logical row length.
+ *   - The caller guarantees operands lie inside the declared ranges and that
+ *     every exact result fits int32.  Outside that contract the output is
+ *     unspecified (integer results are then exact modulo 2^32 as long as the
+ *     operands stay in range).  With QX_FLAG_CHECK_RANGES the device checks
+ *     the operands and qx_plan_status() reports QX_ERR_CONTRACT.
+ *   - Functions return QX_OK or an error code; qx_last_error() gives a one-
+ *     line reason for the most recent failure on the calling thread.
+ */
+#ifndef QX_H
+#define QX_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define QX_VERSION 1
+
+typedef struct qx_plan_s *qx_plan;
+typedef struct CUstream_st *qx_stream; /* identical to cudaStream_t */
+
+typedef enum {
+    QX_OK = 0,
+    QX_ERR_INVALID_ARG = 1,  /* null pointer, bad shape, bad leading dim     */
+    QX_ERR_UNSUPPORTED = 2,  /* alignment, dtype or shape the kernels lack  */
+    QX_ERR_CONTRACT = 3,     /* declared ranges infeasible, or a device range
+                                check found an operand outside its range    */
+    QX_ERR_OOM = 4,          /* workspace allocation failed                 */
+    QX_ERR_CUDA = 5,         /* a CUDA runtime/driver call failed           */
+    QX_ERR_TIMEOUT = 6,      /* a bounded device-side wait expired; the
+                                kernel abandoned its work and exited        */
+    QX_ERR_DEVICE = 7        /* no usable sm_103 device                     */
+} qx_status;
+
+typedef enum { QX_OP_GEMM = 0, QX_OP_CONV2D = 1, QX_OP_ATTN = 2 } qx_op;
+typedef enum { QX_I16 = 0, QX_I32 = 1, QX_F32 = 2 } qx_dtype;
+
+/* Inclusive operand-range contract (Methodology: operand-range contracts
+ * propagate to the operators and decide tiling, packing and accumulation). */
+typedef struct {
+    int64_t lo, hi;
+} qx_range;
+
+/* Ask the device to check every operand against its declared range. */
+#define QX_FLAG_CHECK_RANGES 1u
+
+typedef struct {
+    qx_op op;
+    qx_dtype in_dtype; /* I16 or I32 operands -> int32 output; F32 -> float */
+    /* GEMM: C (M x N) = A (M x K) * B (K x N), all row-major; lda/ldb/ldc are
+     * row pitches in elements (0 means tightly packed). */
+    int64_t M, N, K, lda, ldb, ldc;
+    /* Conv2D: x is NCHW (n, c, h, w), weights KCRS (k_out, c, r, s), output
+     * NCHW (n, k_out, P, Q), P = (h + 2 pad - r) / stride + 1, Q likewise;
+     * cross-correlation, zero padding, no bias, all tightly packed. */
+    int64_t n, c, h, w, k_out, r, s, stride, pad;
+    /* Attention core: Q, K, V and O are L x d, row-major, tightly packed. */
+    int64_t L, d;
+    /* Ranges.  GEMM: range_a = A, range_b = B.  Conv2D: range_a = x,
+     * range_b = weights.  Attention: range_a = Q, range_b = K, range_c = V.
+     * Ignored for F32. */
+    qx_range range_a, range_b, range_c;
+    unsigned flags;
+} qx_plan_desc;
+
+/* How the plan makes one contraction exact on FP16 tensor cores.  An
+ * operand is split into `limbs` balanced digits of `shift` bits (digit i has
+ * weight 2^(i*shift)); every FP16 digit is an exact integer, every limb
+ * product is accumulated in FP32 for at most `chunk_k` terms so that no
+ * partial sum can reach 2^24, and chunks are summed in int32. */
+typedef struct {
+    int limbs_a, shift_a;       /* operand on the tile's row side            */
+    int limbs_b, shift_b;       /* operand on the tile's column side         */
+    int mma_per_kstep;          /* limbs_a * limbs_b tensor-core products    */
+    int64_t chunk_k;            /* K terms per FP32 accumulation chunk       */
+    int64_t n_chunks;           /* ceil(K / chunk_k)                         */
+    int64_t acc_bound;          /* proven max |FP32 partial sum| (< 2^24)    */
+    int64_t k;                  /* contraction length                        */
+} qx_scheme_info;
+
+/* Plan creation (the one-time "setup" of the Methodology paragraph): checks
+ * the descriptor, derives the exact limb scheme from the ranges, allocates
+ * the workspace on `device`, encodes the TMA descriptors on it and caches
+ * the launch arguments.  On success *out owns all of that until
+ * qx_plan_destroy.  Errors: INVALID_ARG, UNSUPPORTED, CONTRACT (no exact
+ * scheme for these ranges), OOM, CUDA, DEVICE. */
+qx_status qx_plan_create(const qx_plan_desc *desc, int device, qx_plan *out);
+
+/* Frees the workspace after synchronising the device.  NULL is a no-op. */
+qx_status qx_plan_destroy(qx_plan plan);
+
+/* Host-only planner: fills up to two scheme records (attention has two
+ * contractions, S = Q K^T then O = S V; other ops have one) without touching
+ * any device.  *count receives the number filled. */
+qx_status qx_plan_query(const qx_plan_desc *desc, qx_scheme_info out[2], int *count);
+
+/* Scheme records of an existing plan (same layout as qx_plan_query). */
+qx_status qx_plan_info(qx_plan plan, qx_scheme_info out[2], int *count);
+
+/* Packed INT16-input / INT32-accumulation GEMM (Abstract; Table 1):
+ * C = A * B with A int16 (M x K, pitch lda), B int16 (K x N, pitch ldb), C
+ * int32 (M x N, pitch ldc).  Plan op GEMM, in_dtype I16. */
+qx_status qx_gemm_i16_i32(qx_plan plan, const int16_t *A, const int16_t *B,
+                          int32_t *C, qx_stream stream);
+
+/* INT32-operand GEMM under the operand-range contract (Methodology; Table 1):
+ * as qx_gemm_i16_i32 with int32 A and B whose values lie in the plan's
+ * declared ranges.  Plan op GEMM, in_dtype I32. */
+qx_status qx_gemm_i32(qx_plan plan, const int32_t *A, const int32_t *B,
+                      int32_t *C, qx_stream stream);
+
+/* GEMM-backed Conv2D (Methodology: convolution through lowering; Table 2):
+ * y = conv(x, w), layouts as in qx_plan_desc.  x and w are int16, int32 or
+ * float per the plan's in_dtype; y is int32 for integer plans and float for
+ * F32 plans.  The lowering happens on load: no patch matrix is written to
+ * device memory. */
+qx_status qx_conv2d_gemm(qx_plan plan, const void *x, const void *w, void *y,
+                         qx_stream stream);
+
+/* Single-head attention core O = (Q K^T) V, no softmax, no scale
+ * (Methodology; Table 2).  Q, K, V, O as in qx_plan_desc, element type per
+ * in_dtype (O is int32 for integer plans, float for F32).  S = Q K^T is
+ * kept on chip; it never goes to device memory. */
+qx_status qx_attn_core(qx_plan plan, const void *Q, const void *K,
+                       const void *V, void *O, qx_stream stream);
+
+/* Synchronises the plan's device, then returns and clears the sticky device
+ * error word (QX_ERR_TIMEOUT or QX_ERR_CONTRACT), or QX_OK. */
+qx_status qx_plan_status(qx_plan plan);
+
+const char *qx_status_string(qx_status status);
+const char *qx_last_error(void);
+int qx_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* QX_H */

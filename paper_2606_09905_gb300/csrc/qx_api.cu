@@ -1,0 +1,652 @@
+// qx_api.cu -- the C ABI (include/qx.h): persistent executors ("plans") that
+// validate a problem once, derive its exact limb scheme from the operand-
+// range contract, allocate the workspace once, encode every TMA descriptor
+// on that workspace once and cache all launch arguments, so each execution
+// call only packs the operands and launches (paper: Methodology, persistent
+// executors that allocate device buffers once and cache uniforms and
+// dispatch metadata).
+#include <cuda.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <string>
+
+#include "qx_internal.h"
+
+namespace qx {
+
+// planner (qx_planner.cu)
+bool make_split(qx_range r, int limbs, int s, Split *out);
+bool plan_contraction(qx_range rn, qx_range rm, int64_t K, Scheme *best);
+void scheme_to_info(const Scheme &s, qx_scheme_info *o);
+// kernels
+bool limb_gemm_supported(int na, int nb);
+int limb_gemm_rows_per_limb(int na);
+cudaError_t limb_gemm_prepare(int na, int nb);
+cudaError_t limb_gemm_launch(int na, int nb, const MmaArgs &a, int grid, cudaStream_t stream);
+cudaError_t attn_prepare();
+cudaError_t attn_launch(const AttnArgs &a, cudaStream_t stream);
+cudaError_t launch_pack_gemm(bool i32, const void *A, const void *B, int64_t lda, int64_t ldb,
+                             int M, int N, int K, int Kp, __half *a_planes, __half *bt_planes,
+                             int na, int shift_a, int nb, int shift_b, int check, qx_range ra,
+                             qx_range rb, int *err, int num_sms, cudaStream_t st);
+cudaError_t launch_pack_conv(bool i32, const void *x, const void *w, int n, int c, int h, int wd,
+                             int k_out, int r, int s, int Cp, __half *x_planes, __half *w_planes,
+                             int nx, int shift_x, int nw, int shift_w, int check, qx_range rx,
+                             qx_range rw, int *err, int num_sms, cudaStream_t st);
+cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int L, int d,
+                             int dp, int Lp, __half *q, __half *k, __half *vt, int int_check,
+                             qx_range rq, qx_range rk, qx_range rv, int *err, int num_sms,
+                             cudaStream_t st);
+
+}  // namespace qx
+
+using namespace qx;
+
+// ------------------------------------------------------------- error text
+static thread_local std::string g_last_error;
+
+static qx_status fail(qx_status st, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return st;
+}
+
+static qx_status cuda_fail(cudaError_t e, const char *what) {
+    cudaGetLastError();  // clear the sticky-free error state
+    return fail(e == cudaErrorMemoryAllocation ? QX_ERR_OOM : QX_ERR_CUDA, "%s: %s", what,
+                cudaGetErrorString(e));
+}
+
+#define QX_CUDA(call, what)                              \
+    do {                                                 \
+        cudaError_t e_ = (call);                         \
+        if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+    } while (0)
+
+// --------------------------------------------------------------- the plan
+struct qx_plan_s {
+    qx_plan_desc desc{};
+    int device = 0;
+    int num_sms = 0;
+    Scheme scheme[2];
+    int n_schemes = 0;
+    void *ws = nullptr;
+    size_t ws_bytes = 0;
+    int *err = nullptr;
+    // GEMM / conv
+    MmaArgs mma{};
+    int grid = 0;
+    __half *planes_n = nullptr, *planes_m = nullptr;
+    int Kp = 0, Cp = 0;
+    // attention
+    AttnArgs attn{};
+    int s_shift = 0, max_keys = 0, dp = 0, Lp = 0;
+    __half *aq = nullptr, *ak = nullptr, *avt = nullptr;
+};
+
+// -------------------------------------------------------- TMA descriptors
+static PFN_cuTensorMapEncodeTiled_v12000 g_encode_tiled = nullptr;
+static PFN_cuTensorMapEncodeIm2col_v12000 g_encode_im2col = nullptr;
+static std::once_flag g_encode_once;
+
+static qx_status load_encoders() {
+    std::call_once(g_encode_once, [] {
+        cudaDriverEntryPointQueryResult q;
+        void *fn = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            g_encode_tiled = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+        fn = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeIm2col", &fn, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            g_encode_im2col = reinterpret_cast<PFN_cuTensorMapEncodeIm2col_v12000>(fn);
+    });
+    if (!g_encode_tiled || !g_encode_im2col)
+        return fail(QX_ERR_CUDA, "driver entry points for TMA descriptor encoding not found");
+    return QX_OK;
+}
+
+// K-major FP16 tensor of `rank` dims (dims[0] innermost), 128-byte swizzle.
+static qx_status encode_tiled(CUtensorMap *map, const void *base, int rank, const uint64_t *dims,
+                              const uint64_t *strides_bytes, const uint32_t *box) {
+    cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    CUresult r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, rank, const_cast<void *>(base),
+                                dims, strides_bytes, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(QX_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", int(r));
+    return QX_OK;
+}
+
+// ------------------------------------------------------------ validation
+static bool bad_range(qx_range r) { return r.lo > r.hi; }
+
+static qx_status check_device(int device, int *num_sms) {
+    int count = 0;
+    cudaError_t e = cudaGetDeviceCount(&count);
+    if (e != cudaSuccess || count <= device || device < 0) {
+        cudaGetLastError();
+        return fail(QX_ERR_DEVICE, "no CUDA device %d (%s)", device,
+                    e == cudaSuccess ? "index out of range" : cudaGetErrorString(e));
+    }
+    cudaDeviceProp prop;
+    QX_CUDA(cudaGetDeviceProperties(&prop, device), "cudaGetDeviceProperties");
+    if (prop.major * 10 + prop.minor != 103)
+        return fail(QX_ERR_DEVICE, "device %d is sm_%d%d; this library is built for sm_103a",
+                    device, prop.major, prop.minor);
+    *num_sms = prop.multiProcessorCount;
+    return QX_OK;
+}
+
+// Scheme(s) of a descriptor; host only.
+static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, int *s_shift,
+                              int *max_keys) {
+    if (!d) return fail(QX_ERR_INVALID_ARG, "null descriptor");
+    if (d->in_dtype != QX_I16 && d->in_dtype != QX_I32 && d->in_dtype != QX_F32)
+        return fail(QX_ERR_INVALID_ARG, "unknown in_dtype %d", int(d->in_dtype));
+    if (d->in_dtype == QX_F32) return fail(QX_ERR_UNSUPPORTED, "FP32 plans are not available");
+    const bool i16 = d->in_dtype == QX_I16;
+    auto range_ok = [&](qx_range r) {
+        if (bad_range(r)) return false;
+        if (i16) return r.lo >= -32768 && r.hi <= 32767;
+        return r.lo >= INT32_MIN && r.hi <= INT32_MAX;
+    };
+    switch (d->op) {
+        case QX_OP_GEMM: {
+            if (d->M < 0 || d->N < 0 || d->K < 0 || d->M > INT32_MAX / 2 || d->N > INT32_MAX / 2 ||
+                d->K > INT32_MAX / 2)
+                return fail(QX_ERR_INVALID_ARG, "GEMM sizes out of range");
+            if (!range_ok(d->range_a) || !range_ok(d->range_b))
+                return fail(QX_ERR_INVALID_ARG, "operand range empty or outside the dtype");
+            // N side = A (rows of C), M side = B (columns of C)
+            if (!plan_contraction(d->range_a, d->range_b, d->K, &out[0]))
+                return fail(QX_ERR_CONTRACT, "no exact limb scheme for these ranges and K");
+            *count = 1;
+            return QX_OK;
+        }
+        case QX_OP_CONV2D: {
+            if (d->n < 1 || d->c < 1 || d->h < 1 || d->w < 1 || d->k_out < 1 || d->r < 1 ||
+                d->s < 1 || d->stride < 1 || d->pad < 0)
+                return fail(QX_ERR_INVALID_ARG, "conv sizes out of range");
+            if (d->h + 2 * d->pad < d->r || d->w + 2 * d->pad < d->s)
+                return fail(QX_ERR_INVALID_ARG, "filter larger than the padded image");
+            if (d->pad > 127 || d->r > 128 || d->s > 128 || d->stride > 8)
+                return fail(QX_ERR_UNSUPPORTED, "conv pad/filter/stride beyond the im2col path");
+            if (!range_ok(d->range_a) || !range_ok(d->range_b))
+                return fail(QX_ERR_INVALID_ARG, "operand range empty or outside the dtype");
+            const int64_t Cp = (d->c + 63) / 64 * 64;
+            // N side = weights (output channels), M side = x (output pixels)
+            if (!plan_contraction(d->range_b, d->range_a, d->r * d->s * Cp, &out[0]))
+                return fail(QX_ERR_CONTRACT, "no exact limb scheme for these ranges");
+            if (out[0].m.limbs > 2) return fail(QX_ERR_UNSUPPORTED, "input needs >2 limbs");
+            *count = 1;
+            return QX_OK;
+        }
+        case QX_OP_ATTN: {
+            if (d->L < 1 || d->d < 1 || d->L > (1 << 24))
+                return fail(QX_ERR_INVALID_ARG, "attention sizes out of range");
+            if (d->d > 128) return fail(QX_ERR_UNSUPPORTED, "attention head size above 128");
+            if (!range_ok(d->range_a) || !range_ok(d->range_b) || !range_ok(d->range_c))
+                return fail(QX_ERR_INVALID_ARG, "operand range empty or outside the dtype");
+            auto mag = [](qx_range r) { return std::max(r.lo < 0 ? -r.lo : r.lo, r.hi < 0 ? -r.hi : r.hi); };
+            const int64_t qm = mag(d->range_a), km = mag(d->range_b), vm = mag(d->range_c);
+            if (qm > kHalfExact || km > kHalfExact || vm > kHalfExact)
+                return fail(QX_ERR_CONTRACT, "attention operands must lie within +-2048");
+            const int64_t smax = d->d * qm * km;
+            if (smax > kAccLimit)
+                return fail(QX_ERR_CONTRACT, "d*max|Q|*max|K| exceeds 2^24");
+            Scheme s0;
+            s0.n.limbs = 1;
+            s0.n.bound[0] = km;
+            s0.m.limbs = 1;
+            s0.m.bound[0] = qm;
+            s0.k = d->d;
+            s0.chunk_kb = (d->d + kBK - 1) / kBK;
+            s0.n_chunks = 1;
+            s0.acc_bound = smax;
+            // S = lo + hi * 2^s; pick the shift that lets a CTA take the most keys
+            int best_s = 0;
+            int64_t best_keys = 0, best_per = 0;
+            Split best_split;
+            for (int s = 1; s <= 12; ++s) {
+                Split sp;
+                if (!make_split(qx_range{-smax, smax}, 2, s, &sp)) continue;
+                const int64_t per = std::max<int64_t>(1, std::max(sp.bound[0], sp.bound[1]) * vm);
+                const int64_t keys = (kAccLimit / per) / 64 * 64;
+                if (keys > best_keys) {
+                    best_keys = keys;
+                    best_s = s;
+                    best_per = per;
+                    best_split = sp;
+                }
+            }
+            if (best_keys < 64) return fail(QX_ERR_CONTRACT, "no exact scheme for S*V");
+            Scheme s1;
+            s1.n = best_split;
+            s1.m.limbs = 1;
+            s1.m.bound[0] = vm;
+            s1.k = d->L;
+            s1.chunk_kb = best_keys / kBK;
+            s1.n_chunks = (d->L + best_keys - 1) / best_keys;
+            s1.acc_bound = best_keys * best_per;
+            out[0] = s0;
+            out[1] = s1;
+            *count = 2;
+            if (s_shift) *s_shift = best_s;
+            if (max_keys) *max_keys = int(std::min<int64_t>(best_keys, INT32_MAX / 2));
+            return QX_OK;
+        }
+        default:
+            return fail(QX_ERR_INVALID_ARG, "unknown op %d", int(d->op));
+    }
+}
+
+static size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
+
+// ----------------------------------------------------------- device scope
+struct DeviceScope {
+    int prev = -1;
+    bool changed = false;
+    cudaError_t enter(int dev) {
+        cudaError_t e = cudaGetDevice(&prev);
+        if (e != cudaSuccess) return e;
+        if (prev != dev) {
+            changed = true;
+            return cudaSetDevice(dev);
+        }
+        return cudaSuccess;
+    }
+    ~DeviceScope() {
+        if (changed) cudaSetDevice(prev);
+    }
+};
+
+// ------------------------------------------------------------ plan build
+static qx_status build_gemm(qx_plan p) {
+    const qx_plan_desc &d = p->desc;
+    const Scheme &s = p->scheme[0];
+    const int na = s.n.limbs, nb = s.m.limbs;
+    const int mr = limb_gemm_rows_per_limb(na);
+    p->Kp = int((d.K + 7) / 8 * 8);
+    const size_t a_bytes = size_t(na) * d.M * p->Kp * 2;
+    const size_t b_bytes = size_t(nb) * d.N * p->Kp * 2;
+    p->ws_bytes = 256 + align256(a_bytes) + align256(b_bytes);
+    QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
+    p->err = static_cast<int *>(p->ws);
+    p->planes_n = reinterpret_cast<__half *>(static_cast<char *>(p->ws) + 256);
+    p->planes_m = reinterpret_cast<__half *>(static_cast<char *>(p->ws) + 256 + align256(a_bytes));
+    QX_CUDA(cudaMemset(p->err, 0, sizeof(int)), "error word reset");
+
+    MmaArgs &a = p->mma;
+    memset(&a, 0, sizeof a);
+    if (d.M > 0 && d.N > 0 && d.K > 0) {
+        for (int j = 0; j < nb; ++j) {
+            const uint64_t dims[2] = {uint64_t(d.K), uint64_t(d.N)};
+            const uint64_t str[1] = {uint64_t(p->Kp) * 2};
+            const uint32_t box[2] = {kBK, kBM};
+            qx_status st = encode_tiled(&a.tm_m[j], p->planes_m + size_t(j) * d.N * p->Kp, 2,
+                                        dims, str, box);
+            if (st != QX_OK) return st;
+        }
+        const uint64_t dims[3] = {uint64_t(d.K), uint64_t(d.M), uint64_t(na)};
+        const uint64_t str[2] = {uint64_t(p->Kp) * 2, uint64_t(d.M) * p->Kp * 2};
+        const uint32_t box[3] = {kBK, uint32_t(mr), uint32_t(na)};
+        qx_status st = encode_tiled(&a.tm_n, p->planes_n, 3, dims, str, box);
+        if (st != QX_OK) return st;
+    }
+    a.err = p->err;
+    a.out_row_stride = d.ldc;
+    a.mode = 0;
+    a.m_extent = int(d.N);
+    a.n_extent = int(d.M);
+    a.kblocks = int((d.K + kBK - 1) / kBK);
+    a.chunk_kb = int(s.chunk_kb);
+    a.tiles_m = int((d.N + kBM - 1) / kBM);
+    a.tiles_n = int((d.M + mr - 1) / mr);
+    a.group_n = std::max(1, std::min(16, a.tiles_n));
+    a.shift_n = s.n.shift;
+    a.shift_m = s.m.shift;
+    const int tiles = a.tiles_m * a.tiles_n;
+    p->grid = std::max(1, std::min(tiles, p->num_sms));
+    QX_CUDA(limb_gemm_prepare(na, nb), "kernel attributes");
+    return QX_OK;
+}
+
+static qx_status build_conv(qx_plan p) {
+    const qx_plan_desc &d = p->desc;
+    const Scheme &s = p->scheme[0];
+    const int nw = s.n.limbs, nx = s.m.limbs;
+    const int mr = limb_gemm_rows_per_limb(nw);
+    const int64_t P = (d.h + 2 * d.pad - d.r) / d.stride + 1;
+    const int64_t Q = (d.w + 2 * d.pad - d.s) / d.stride + 1;
+    p->Cp = int((d.c + 63) / 64 * 64);
+    const size_t x_bytes = size_t(nx) * d.n * d.h * d.w * p->Cp * 2;
+    const size_t w_bytes = size_t(nw) * d.k_out * d.r * d.s * p->Cp * 2;
+    p->ws_bytes = 256 + align256(x_bytes) + align256(w_bytes);
+    QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
+    p->err = static_cast<int *>(p->ws);
+    p->planes_m = reinterpret_cast<__half *>(static_cast<char *>(p->ws) + 256);
+    p->planes_n = reinterpret_cast<__half *>(static_cast<char *>(p->ws) + 256 + align256(x_bytes));
+    QX_CUDA(cudaMemset(p->err, 0, sizeof(int)), "error word reset");
+
+    MmaArgs &a = p->mma;
+    memset(&a, 0, sizeof a);
+    for (int j = 0; j < nx; ++j) {
+        const cuuint64_t dims[4] = {cuuint64_t(p->Cp), cuuint64_t(d.w), cuuint64_t(d.h),
+                                    cuuint64_t(d.n)};
+        const cuuint64_t str[3] = {cuuint64_t(p->Cp) * 2, cuuint64_t(d.w) * p->Cp * 2,
+                                   cuuint64_t(d.h) * d.w * p->Cp * 2};
+        const int lower[2] = {int(-d.pad), int(-d.pad)};
+        const int upper[2] = {int(d.pad - (d.s - 1)), int(d.pad - (d.r - 1))};
+        const cuuint32_t estr[4] = {1, cuuint32_t(d.stride), cuuint32_t(d.stride), 1};
+        CUresult r = g_encode_im2col(&a.tm_m[j], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4,
+                                     p->planes_m + size_t(j) * d.n * d.h * d.w * p->Cp, dims, str,
+                                     lower, upper, kBK, kBM, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS)
+            return fail(QX_ERR_UNSUPPORTED, "cuTensorMapEncodeIm2col failed (%d)", int(r));
+    }
+    const int64_t Kg = d.r * d.s * p->Cp;
+    {
+        const uint64_t dims[3] = {uint64_t(Kg), uint64_t(d.k_out), uint64_t(nw)};
+        const uint64_t str[2] = {uint64_t(Kg) * 2, uint64_t(d.k_out) * Kg * 2};
+        const uint32_t box[3] = {kBK, uint32_t(mr), uint32_t(nw)};
+        qx_status st = encode_tiled(&a.tm_n, p->planes_n, 3, dims, str, box);
+        if (st != QX_OK) return st;
+    }
+    a.err = p->err;
+    a.out_row_stride = P * Q;
+    a.mode = 1;
+    a.m_extent = int(d.n * P * Q);
+    a.n_extent = int(d.k_out);
+    a.kblocks = int(Kg / kBK);
+    a.chunk_kb = int(s.chunk_kb);
+    a.tiles_m = int((a.m_extent + kBM - 1) / kBM);
+    a.tiles_n = int((d.k_out + mr - 1) / mr);
+    a.group_n = std::max(1, std::min(16, a.tiles_n));
+    a.shift_n = s.n.shift;
+    a.shift_m = s.m.shift;
+    a.c_blocks = p->Cp / kBK;
+    a.S = int(d.s);
+    a.Q = int(Q);
+    a.PQ = int(P * Q);
+    a.stride = int(d.stride);
+    a.pad = int(d.pad);
+    a.k_out = int(d.k_out);
+    const int tiles = a.tiles_m * a.tiles_n;
+    p->grid = std::max(1, std::min(tiles, p->num_sms));
+    QX_CUDA(limb_gemm_prepare(nw, nx), "kernel attributes");
+    return QX_OK;
+}
+
+static qx_status build_attn(qx_plan p) {
+    const qx_plan_desc &d = p->desc;
+    p->dp = d.d <= 64 ? 64 : 128;
+    p->Lp = int((d.L + 7) / 8 * 8);
+    const size_t qk_bytes = size_t(d.L) * p->dp * 2;
+    const size_t vt_bytes = size_t(p->dp) * p->Lp * 2;
+    p->ws_bytes = 256 + 2 * align256(qk_bytes) + align256(vt_bytes);
+    QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
+    char *base = static_cast<char *>(p->ws);
+    p->err = reinterpret_cast<int *>(base);
+    p->aq = reinterpret_cast<__half *>(base + 256);
+    p->ak = reinterpret_cast<__half *>(base + 256 + align256(qk_bytes));
+    p->avt = reinterpret_cast<__half *>(base + 256 + 2 * align256(qk_bytes));
+    QX_CUDA(cudaMemset(p->err, 0, sizeof(int)), "error word reset");
+
+    AttnArgs &a = p->attn;
+    memset(&a, 0, sizeof a);
+    {
+        const uint64_t dims[2] = {uint64_t(p->dp), uint64_t(d.L)};
+        const uint64_t str[1] = {uint64_t(p->dp) * 2};
+        const uint32_t boxq[2] = {64, 128};
+        const uint32_t boxk[2] = {64, 64};
+        qx_status st = encode_tiled(&a.tm_q, p->aq, 2, dims, str, boxq);
+        if (st != QX_OK) return st;
+        st = encode_tiled(&a.tm_k, p->ak, 2, dims, str, boxk);
+        if (st != QX_OK) return st;
+    }
+    {
+        const uint64_t dims[2] = {uint64_t(d.L), uint64_t(p->dp)};
+        const uint64_t str[1] = {uint64_t(p->Lp) * 2};
+        const uint32_t box[2] = {64, 128};
+        qx_status st = encode_tiled(&a.tm_vt, p->avt, 2, dims, str, box);
+        if (st != QX_OK) return st;
+    }
+    a.err = p->err;
+    a.L = int(d.L);
+    a.d = int(d.d);
+    a.q_tiles = int((d.L + 127) / 128);
+    const int key_blocks = int((d.L + 63) / 64);
+    const int max_blocks = std::max(1, p->max_keys / 64);
+    int splits = std::max(1, std::min(key_blocks, (p->num_sms + a.q_tiles - 1) / a.q_tiles));
+    int per = (key_blocks + splits - 1) / splits;
+    if (per > max_blocks) {
+        per = max_blocks;
+        splits = (key_blocks + per - 1) / per;
+    }
+    splits = (key_blocks + per - 1) / per;
+    a.key_splits = splits;
+    a.keys_per_split = per * 64;
+    a.s_shift = p->s_shift;
+    a.o_chunk_kb = max_blocks;
+    QX_CUDA(attn_prepare(), "kernel attributes");
+    return QX_OK;
+}
+
+// ================================================================ C ABI
+extern "C" {
+
+int qx_version(void) { return QX_VERSION; }
+
+const char *qx_last_error(void) { return g_last_error.c_str(); }
+
+const char *qx_status_string(qx_status s) {
+    switch (s) {
+        case QX_OK: return "ok";
+        case QX_ERR_INVALID_ARG: return "invalid argument";
+        case QX_ERR_UNSUPPORTED: return "unsupported";
+        case QX_ERR_CONTRACT: return "operand-range contract";
+        case QX_ERR_OOM: return "out of device memory";
+        case QX_ERR_CUDA: return "CUDA error";
+        case QX_ERR_TIMEOUT: return "device wait timed out";
+        case QX_ERR_DEVICE: return "no usable device";
+    }
+    return "unknown status";
+}
+
+qx_status qx_plan_query(const qx_plan_desc *desc, qx_scheme_info out[2], int *count) {
+    if (!out || !count) return fail(QX_ERR_INVALID_ARG, "null output");
+    Scheme s[2];
+    int n = 0;
+    qx_status st = plan_schemes(desc, s, &n, nullptr, nullptr);
+    if (st != QX_OK) return st;
+    for (int i = 0; i < n; ++i) scheme_to_info(s[i], &out[i]);
+    *count = n;
+    return QX_OK;
+}
+
+qx_status qx_plan_create(const qx_plan_desc *desc, int device, qx_plan *out) {
+    if (!out) return fail(QX_ERR_INVALID_ARG, "null plan output");
+    *out = nullptr;
+    if (!desc) return fail(QX_ERR_INVALID_ARG, "null descriptor");
+    qx_plan_desc d = *desc;
+    if (d.op == QX_OP_GEMM) {
+        if (d.lda == 0) d.lda = d.K;
+        if (d.ldb == 0) d.ldb = d.N;
+        if (d.ldc == 0) d.ldc = d.N;
+        if (d.lda < d.K || d.ldb < d.N || d.ldc < d.N)
+            return fail(QX_ERR_INVALID_ARG, "leading dimension shorter than the row");
+    }
+    qx_plan_s tmp;
+    int s_shift = 0, max_keys = 0;
+    qx_status st = plan_schemes(&d, tmp.scheme, &tmp.n_schemes, &s_shift, &max_keys);
+    if (st != QX_OK) return st;
+    int num_sms = 0;
+    st = check_device(device, &num_sms);
+    if (st != QX_OK) return st;
+    st = load_encoders();
+    if (st != QX_OK) return st;
+
+    DeviceScope scope;
+    QX_CUDA(scope.enter(device), "cudaSetDevice");
+    qx_plan p = new (std::nothrow) qx_plan_s();
+    if (!p) return fail(QX_ERR_OOM, "host allocation");
+    p->desc = d;
+    p->device = device;
+    p->num_sms = num_sms;
+    p->n_schemes = tmp.n_schemes;
+    p->scheme[0] = tmp.scheme[0];
+    p->scheme[1] = tmp.scheme[1];
+    p->s_shift = s_shift;
+    p->max_keys = max_keys;
+    switch (d.op) {
+        case QX_OP_GEMM: st = build_gemm(p); break;
+        case QX_OP_CONV2D: st = build_conv(p); break;
+        case QX_OP_ATTN: st = build_attn(p); break;
+        default: st = fail(QX_ERR_INVALID_ARG, "unknown op");
+    }
+    if (st != QX_OK) {
+        if (p->ws) cudaFree(p->ws);
+        delete p;
+        return st;
+    }
+    *out = p;
+    return QX_OK;
+}
+
+qx_status qx_plan_destroy(qx_plan p) {
+    if (!p) return QX_OK;
+    qx_status st = QX_OK;
+    {
+        DeviceScope scope;
+        if (scope.enter(p->device) == cudaSuccess) {
+            cudaError_t e = cudaDeviceSynchronize();
+            if (e != cudaSuccess) st = cuda_fail(e, "cudaDeviceSynchronize");
+            if (p->ws) cudaFree(p->ws);
+        }
+    }
+    delete p;
+    return st;
+}
+
+qx_status qx_plan_info(qx_plan p, qx_scheme_info out[2], int *count) {
+    if (!p || !out || !count) return fail(QX_ERR_INVALID_ARG, "null argument");
+    for (int i = 0; i < p->n_schemes; ++i) scheme_to_info(p->scheme[i], &out[i]);
+    *count = p->n_schemes;
+    return QX_OK;
+}
+
+qx_status qx_plan_status(qx_plan p) {
+    if (!p) return fail(QX_ERR_INVALID_ARG, "null plan");
+    DeviceScope scope;
+    QX_CUDA(scope.enter(p->device), "cudaSetDevice");
+    QX_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+    int word = 0;
+    QX_CUDA(cudaMemcpy(&word, p->err, sizeof word, cudaMemcpyDeviceToHost), "error word read");
+    QX_CUDA(cudaMemset(p->err, 0, sizeof word), "error word reset");
+    if (word == 0) return QX_OK;
+    return fail(qx_status(word), "device reported: %s", qx_status_string(qx_status(word)));
+}
+
+static bool aligned16(const void *ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
+
+static qx_status run_gemm(qx_plan p, const void *A, const void *B, int32_t *C, cudaStream_t stream,
+                          qx_dtype want) {
+    if (!p) return fail(QX_ERR_INVALID_ARG, "null plan");
+    const qx_plan_desc &d = p->desc;
+    if (d.op != QX_OP_GEMM || d.in_dtype != want)
+        return fail(QX_ERR_INVALID_ARG, "plan is not a %s GEMM plan", want == QX_I16 ? "I16" : "I32");
+    if (d.M == 0 || d.N == 0) return QX_OK;
+    if (!C || (d.K > 0 && (!A || !B))) return fail(QX_ERR_INVALID_ARG, "null operand");
+    if (!aligned16(C) || (d.K > 0 && (!aligned16(A) || !aligned16(B))))
+        return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+    DeviceScope scope;
+    QX_CUDA(scope.enter(p->device), "cudaSetDevice");
+    if (d.K == 0) {
+        QX_CUDA(cudaMemset2DAsync(C, size_t(d.ldc) * 4, 0, size_t(d.N) * 4, size_t(d.M), stream),
+                "zero output");
+        return QX_OK;
+    }
+    const Scheme &s = p->scheme[0];
+    QX_CUDA(launch_pack_gemm(want == QX_I32, A, B, d.lda, d.ldb, int(d.M), int(d.N), int(d.K),
+                             p->Kp, p->planes_n, p->planes_m, s.n.limbs, s.n.shift, s.m.limbs,
+                             s.m.shift, (d.flags & QX_FLAG_CHECK_RANGES) ? 1 : 0, d.range_a,
+                             d.range_b, p->err, p->num_sms, stream),
+            "operand packing launch");
+    MmaArgs a = p->mma;
+    a.out = C;
+    QX_CUDA(limb_gemm_launch(s.n.limbs, s.m.limbs, a, p->grid, stream), "limb GEMM launch");
+    return QX_OK;
+}
+
+qx_status qx_gemm_i16_i32(qx_plan p, const int16_t *A, const int16_t *B, int32_t *C,
+                          qx_stream stream) {
+    return run_gemm(p, A, B, C, reinterpret_cast<cudaStream_t>(stream), QX_I16);
+}
+
+qx_status qx_gemm_i32(qx_plan p, const int32_t *A, const int32_t *B, int32_t *C, qx_stream stream) {
+    return run_gemm(p, A, B, C, reinterpret_cast<cudaStream_t>(stream), QX_I32);
+}
+
+qx_status qx_conv2d_gemm(qx_plan p, const void *x, const void *w, void *y, qx_stream stream) {
+    if (!p) return fail(QX_ERR_INVALID_ARG, "null plan");
+    const qx_plan_desc &d = p->desc;
+    if (d.op != QX_OP_CONV2D) return fail(QX_ERR_INVALID_ARG, "plan is not a conv plan");
+    if (!x || !w || !y) return fail(QX_ERR_INVALID_ARG, "null operand");
+    if (!aligned16(x) || !aligned16(w) || !aligned16(y))
+        return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+    DeviceScope scope;
+    QX_CUDA(scope.enter(p->device), "cudaSetDevice");
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const Scheme &s = p->scheme[0];
+    QX_CUDA(launch_pack_conv(d.in_dtype == QX_I32, x, w, int(d.n), int(d.c), int(d.h), int(d.w),
+                             int(d.k_out), int(d.r), int(d.s), p->Cp, p->planes_m, p->planes_n,
+                             s.m.limbs, s.m.shift, s.n.limbs, s.n.shift,
+                             (d.flags & QX_FLAG_CHECK_RANGES) ? 1 : 0, d.range_a, d.range_b,
+                             p->err, p->num_sms, st),
+            "operand packing launch");
+    MmaArgs a = p->mma;
+    a.out = static_cast<int32_t *>(y);
+    QX_CUDA(limb_gemm_launch(s.n.limbs, s.m.limbs, a, p->grid, st), "conv launch");
+    return QX_OK;
+}
+
+qx_status qx_attn_core(qx_plan p, const void *Q, const void *K, const void *V, void *O,
+                       qx_stream stream) {
+    if (!p) return fail(QX_ERR_INVALID_ARG, "null plan");
+    const qx_plan_desc &d = p->desc;
+    if (d.op != QX_OP_ATTN) return fail(QX_ERR_INVALID_ARG, "plan is not an attention plan");
+    if (!Q || !K || !V || !O) return fail(QX_ERR_INVALID_ARG, "null operand");
+    if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
+        return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+    DeviceScope scope;
+    QX_CUDA(scope.enter(p->device), "cudaSetDevice");
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    QX_CUDA(cudaMemsetAsync(O, 0, size_t(d.L) * d.d * 4, st), "zero output");
+    QX_CUDA(launch_pack_attn(d.in_dtype == QX_I32, Q, K, V, int(d.L), int(d.d), p->dp, p->Lp,
+                             p->aq, p->ak, p->avt, (d.flags & QX_FLAG_CHECK_RANGES) ? 1 : 0,
+                             d.range_a, d.range_b, d.range_c, p->err, p->num_sms, st),
+            "operand packing launch");
+    AttnArgs a = p->attn;
+    a.out = static_cast<int32_t *>(O);
+    QX_CUDA(attn_launch(a, st), "attention launch");
+    return QX_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,75 @@
+// qx_internal.h -- definitions shared by the host API and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "../../include/qx.h"
+
+namespace qx {
+
+// Largest |partial sum| an FP32 accumulator may reach and stay exact: every
+// integer of magnitude <= 2^24 is representable in binary32.
+constexpr int64_t kAccLimit = int64_t(1) << 24;
+// Largest |integer| an FP16 limb may hold exactly (11-bit significand).
+constexpr int64_t kHalfExact = 2048;
+// K extent of one pipeline stage: 64 FP16 values = one 128-byte swizzle row.
+constexpr int kBK = 64;
+// Rows of the tile on the MMA's M side (TMEM lanes).
+constexpr int kBM = 128;
+
+// Device error word values (the same numbers as qx_status).
+constexpr int kErrContract = QX_ERR_CONTRACT;
+constexpr int kErrTimeout = QX_ERR_TIMEOUT;
+
+// One operand's split into balanced base-2^shift digits.
+struct Split {
+    int limbs = 1;
+    int shift = 0;
+    int64_t bound[4] = {0, 0, 0, 0};   // max |digit i| over the declared range
+};
+
+// The exact scheme for one contraction.  "n" is the operand whose limbs are
+// stacked along the MMA's N dimension; "m" the operand on the M side, whose
+// limbs get accumulators of their own.
+struct Scheme {
+    Split n, m;
+    int64_t k = 0;
+    int64_t chunk_kb = 1;   // k-blocks (of kBK) per FP32 chunk
+    int64_t n_chunks = 0;
+    int64_t acc_bound = 0;  // max |partial| an accumulator can reach in a chunk
+};
+
+// Kernel arguments of the tiled limb GEMM, cached in the plan.
+struct MmaArgs {
+    CUtensorMap tm_m[2];      // M-side operand, one map per limb
+    CUtensorMap tm_n;         // N-side operand: 3-D (k, row, limb)
+    int32_t *out;             // set per call
+    int *err;                 // device error word
+    int64_t out_row_stride;   // elements between consecutive N-side rows
+    int mode;                 // 0 = GEMM, 1 = conv (im2col M side, NCHW out)
+    int m_extent;             // M-side rows (GEMM: N columns of C; conv: pixels)
+    int n_extent;             // N-side rows (GEMM: M rows of C; conv: k_out)
+    int kblocks;              // ceil(K / kBK)
+    int chunk_kb;             // k-blocks per FP32 accumulation chunk
+    int tiles_m, tiles_n, group_n;
+    int shift_n, shift_m;     // digit widths of the N-side / M-side limbs
+    // conv geometry (mode 1)
+    int c_blocks, S, Q, PQ, stride, pad, k_out;
+};
+
+// Kernel arguments of the fused attention core.
+struct AttnArgs {
+    CUtensorMap tm_q;         // Q   (L x d) fp16, 2-D
+    CUtensorMap tm_k;         // K   (L x d) fp16, 2-D
+    CUtensorMap tm_vt;        // V^T (d x L) fp16, 2-D (K-major for the 2nd MMA)
+    int32_t *out;             // O (L x d) int32, zeroed before the launch
+    int *err;
+    int L, d;
+    int q_tiles, key_splits, keys_per_split;
+    int s_shift;              // digit width of the S limbs
+    int o_chunk_kb;           // key-blocks per FP32 chunk of the second product
+};
+
+}  // namespace qx

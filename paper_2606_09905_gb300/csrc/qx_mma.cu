@@ -1,0 +1,351 @@
+// qx_mma.cu -- the tiled limb GEMM: the one substrate that the integer GEMMs
+// and the GEMM-backed Conv2D share (paper: Methodology, "reuse a tiled
+// matrix-multiplication substrate"; Table 1; Table 2 Conv2D rows).
+//
+// Exactness.  Integer operands arrive as FP16 limb planes (balanced digits,
+// every digit an exact FP16 integer).  tcgen05.mma kind::f16 multiplies limb
+// tiles and accumulates in FP32 in tensor memory.  The planner bounds every
+// accumulator's partial sums by 2^24 over a chunk of k-blocks, so each FP32
+// value is an exact integer; at each chunk end the epilogue converts the
+// accumulators to int32 (exact), shifts each by its limb weight and adds them
+// into int32 registers with wrapping arithmetic.  The result is the exact
+// product modulo 2^32, i.e. the exact int32 result under the contract.
+//
+// Orientation.  The MMA's M side (128 TMEM lanes) is the output's contiguous
+// dimension: columns of C for the GEMM (B^T tile), output pixels for the conv
+// (im2col tile).  The N side stacks the limbs of the other operand (rows of
+// A, or output channels of the weights): N = limbs * MR.  So one MMA computes
+// every limb of that operand at once, and each epilogue thread owns one
+// output column, which makes every warp store 32 consecutive int32 values.
+//
+// Roles (one CTA per SM, persistent over output tiles):
+//   warp 0      TMA producer (one thread): stage ring of `STAGES` buffers
+//   warp 1      TMEM owner and MMA issuer (one thread)
+//   warps 2..9  epilogue: two warps per TMEM lane quarter, each owning half
+//               of the N-side rows; running int32 sums live in registers.
+// Accumulators are double-buffered in TMEM whenever they fit in 256 columns,
+// so the epilogue drains chunk c while the tensor cores run chunk c + 1.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "qx_device.cuh"
+#include "qx_internal.h"
+
+namespace qx {
+
+template <int NA, int NB>
+struct TileCfg {
+    static constexpr int MR = NA <= 2 ? 128 : 64;   // N-side rows per limb
+    static constexpr int UN = NA * MR;              // MMA N
+    static constexpr int M_TILE = kBM * 128;        // bytes of one M-side limb tile
+    static constexpr int N_TILE = UN * 128;         // bytes of the stacked N-side tile
+    static constexpr int STAGE = NB * M_TILE + N_TILE;
+    static constexpr int STAGES_FIT = (200 * 1024) / STAGE;
+    static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
+    static constexpr int ACC_COLS = NB * UN;        // TMEM columns per accumulator set
+    static constexpr int NBUF = ACC_COLS <= 256 ? 2 : 1;
+    static constexpr int TMEM_NEED = ACC_COLS * NBUF;
+    static constexpr int TMEM_COLS = TMEM_NEED <= 32    ? 32
+                                     : TMEM_NEED <= 64  ? 64
+                                     : TMEM_NEED <= 128 ? 128
+                                     : TMEM_NEED <= 256 ? 256
+                                                        : 512;
+    static constexpr int RPT = MR / 2;              // N-side rows per epilogue thread
+    static constexpr uint32_t IDESC = make_idesc(kBM, UN, 0);
+    static constexpr int BAR_BYTES = 256;
+    static constexpr int SMEM = STAGES * STAGE + BAR_BYTES + 1024;
+    static constexpr int THREADS = 320;
+    static_assert(UN % 16 == 0 && UN >= 16 && UN <= 256, "MMA N out of range");
+    static_assert(TMEM_NEED <= 512, "accumulators exceed tensor memory");
+    static_assert(RPT % 32 == 0, "epilogue works in 32-column TMEM loads");
+};
+
+// Tile order: groups of `group_n` N-side tiles, M-side tiles inside a group,
+// so the CTAs resident at one time share operand tiles through L2.
+__device__ __forceinline__ void tile_coords(int t, const MmaArgs &a, int &tm, int &tn) {
+    const int per_group = a.group_n * a.tiles_m;
+    const int g = t / per_group;
+    const int first = g * a.group_n;
+    const int gs = min(a.group_n, a.tiles_n - first);
+    const int r = t - g * per_group;
+    tn = first + r % gs;
+    tm = r / gs;
+}
+
+template <int NA, int NB>
+__global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant__ MmaArgs a) {
+    using T = TileCfg<NA, NB>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + T::STAGES * T::STAGE);
+    uint64_t *empty = full + T::STAGES;
+    uint64_t *acc_full = empty + T::STAGES;
+    uint64_t *acc_empty = acc_full + 2;
+    uint64_t *tail = acc_empty + 2;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(tail + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int ntiles = a.tiles_m * a.tiles_n;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < T::STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], 8);
+        }
+        mbar_init(tail, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, T::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ------------------------------------------------ TMA producer
+            tma_prefetch(&a.tm_m[0]);
+            if (NB > 1) tma_prefetch(&a.tm_m[1]);
+            tma_prefetch(&a.tm_n);
+            int stage = 0;
+            uint32_t phase = 0;
+            long long issued = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+                int tm, tn;
+                tile_coords(t, a, tm, tn);
+                int img = 0, oh = 0, ow = 0;
+                if (a.mode == 1) {
+                    const int p0 = tm * kBM;
+                    img = p0 / a.PQ;
+                    const int rem = p0 - img * a.PQ;
+                    oh = rem / a.Q;
+                    ow = rem - oh * a.Q;
+                }
+                for (int kb = 0; kb < a.kblocks; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, a.err)) {
+                        ok = false;
+                        break;
+                    }
+                    uint8_t *st = smem + stage * T::STAGE;
+                    mbar_expect_tx(&full[stage], T::STAGE);
+                    if (a.mode == 0) {
+#pragma unroll
+                        for (int j = 0; j < NB; ++j)
+                            tma_load_2d(st + j * T::M_TILE, &a.tm_m[j], &full[stage], kb * kBK,
+                                        tm * kBM);
+                    } else {
+                        const int tap = kb / a.c_blocks;
+                        const int cb = kb - tap * a.c_blocks;
+                        const int r = tap / a.S;
+                        const int s = tap - r * a.S;
+#pragma unroll
+                        for (int j = 0; j < NB; ++j)
+                            tma_load_im2col_4d(st + j * T::M_TILE, &a.tm_m[j], &full[stage],
+                                               cb * kBK, ow * a.stride - a.pad,
+                                               oh * a.stride - a.pad, img, uint16_t(s),
+                                               uint16_t(r));
+                    }
+                    tma_load_3d(st + NB * T::M_TILE, &a.tm_n, &full[stage], kb * kBK,
+                                tn * T::MR, 0);
+                    ++issued;
+                    if (++stage == T::STAGES) {
+                        stage = 0;
+                        phase ^= 1;
+                    }
+                }
+            }
+            if (ok) {
+                // Every stage must be released by the MMA before the CTA exits,
+                // so that no commit lands on the barriers of a later CTA.
+                for (int i = 0; i < T::STAGES; ++i) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, a.err)) break;
+                    if (++stage == T::STAGES) {
+                        stage = 0;
+                        phase ^= 1;
+                    }
+                }
+            }
+            if (*abort_flag) {
+                // Let every copy already issued land before shared memory goes.
+                for (int s = 0; s < T::STAGES; ++s) {
+                    const long long uses =
+                        issued / T::STAGES + (s < issued % T::STAGES ? 1 : 0);
+                    if (uses > 0) mbar_wait_drain(&full[s], uint32_t((uses - 1) & 1));
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // -------------------------------------------------- MMA issuer
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t acc_it = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+                for (int kb0 = 0; kb0 < a.kblocks; kb0 += a.chunk_kb) {
+                    const int kb1 = min(kb0 + a.chunk_kb, a.kblocks);
+                    const uint32_t buf = T::NBUF == 2 ? (acc_it & 1u) : 0u;
+                    const uint32_t apar = T::NBUF == 2 ? ((acc_it >> 1) & 1u) : (acc_it & 1u);
+                    if (!mbar_wait(&acc_empty[buf], apar ^ 1, abort_flag, a.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t d0 = tmem_base + buf * T::ACC_COLS;
+                    for (int kb = kb0; kb < kb1; ++kb) {
+                        if (!mbar_wait(&full[stage], phase, abort_flag, a.err)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t sbase = smem_addr(smem + stage * T::STAGE);
+#pragma unroll
+                        for (int kk = 0; kk < kBK / 16; ++kk) {
+                            const uint64_t bdesc = make_sdesc(sbase + NB * T::M_TILE + kk * 32);
+#pragma unroll
+                            for (int j = 0; j < NB; ++j) {
+                                const uint64_t adesc = make_sdesc(sbase + j * T::M_TILE + kk * 32);
+                                mma_f16(d0 + j * T::UN, adesc, bdesc, T::IDESC,
+                                        (kb > kb0 || kk > 0) ? 1u : 0u);
+                            }
+                        }
+                        tc_commit(&empty[stage]);
+                        if (++stage == T::STAGES) {
+                            stage = 0;
+                            phase ^= 1;
+                        }
+                    }
+                    if (!ok) break;
+                    tc_commit(&acc_full[buf]);
+                    ++acc_it;
+                }
+            }
+            if (!ok) {
+                // MMAs already issued must finish before TMEM is released.
+                tc_commit(tail);
+                mbar_wait_drain(tail, 0);
+            }
+        }
+    } else {
+        // ------------------------------------------------------ epilogue
+        const int q = warp & 3;             // TMEM lane quarter this warp may read
+        const int hh = (warp - 2) >> 2;     // which half of the N-side rows
+        uint32_t acc_it = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+            int tm, tn;
+            tile_coords(t, a, tm, tn);
+            uint32_t acc[T::RPT];
+#pragma unroll
+            for (int r = 0; r < T::RPT; ++r) acc[r] = 0u;
+            for (int kb0 = 0; kb0 < a.kblocks; kb0 += a.chunk_kb) {
+                const uint32_t buf = T::NBUF == 2 ? (acc_it & 1u) : 0u;
+                const uint32_t apar = T::NBUF == 2 ? ((acc_it >> 1) & 1u) : (acc_it & 1u);
+                if (!mbar_wait(&acc_full[buf], apar, abort_flag, a.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t tb =
+                    tmem_base + (uint32_t(q * 32) << 16) + buf * T::ACC_COLS + hh * T::RPT;
+#pragma unroll
+                for (int j = 0; j < NB; ++j) {
+#pragma unroll
+                    for (int i = 0; i < NA; ++i) {
+                        const int sh = i * a.shift_n + j * a.shift_m;
+#pragma unroll
+                        for (int p = 0; p < T::RPT / 32; ++p) {
+                            uint32_t v[32];
+                            tmem_ld32(tb + j * T::UN + i * T::MR + p * 32, v);
+                            tmem_wait_ld(v);
+#pragma unroll
+                            for (int x = 0; x < 32; ++x)
+                                acc[p * 32 + x] +=
+                                    uint32_t(__float2int_rn(__uint_as_float(v[x]))) << sh;
+                        }
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&acc_empty[buf]);
+                ++acc_it;
+            }
+            if (!ok) break;
+            const int mrow = tm * kBM + q * 32 + lane;
+            const bool lane_ok = mrow < a.m_extent;
+            int64_t lane_off = mrow;
+            if (a.mode == 1) {
+                const int img = mrow / a.PQ;
+                lane_off = int64_t(img) * a.k_out * a.PQ + (mrow - img * a.PQ);
+            }
+            const int nrow0 = tn * T::MR + hh * T::RPT;
+            int32_t *o = a.out + lane_off + int64_t(nrow0) * a.out_row_stride;
+#pragma unroll
+            for (int r = 0; r < T::RPT; ++r) {
+                if (lane_ok && nrow0 + r < a.n_extent)
+                    o[int64_t(r) * a.out_row_stride] = int32_t(acc[r]);
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, T::TMEM_COLS);
+    }
+}
+
+// ------------------------------------------------------------------- host
+template <int NA, int NB>
+static cudaError_t prepare_t() {
+    return cudaFuncSetAttribute(limb_gemm_kernel<NA, NB>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, TileCfg<NA, NB>::SMEM);
+}
+
+template <int NA, int NB>
+static cudaError_t launch_t(const MmaArgs &a, int grid, cudaStream_t stream) {
+    limb_gemm_kernel<NA, NB><<<grid, TileCfg<NA, NB>::THREADS, TileCfg<NA, NB>::SMEM, stream>>>(a);
+    return cudaGetLastError();
+}
+
+#define QX_LIMB_DISPATCH(FN, ...)                                          \
+    switch (na * 10 + nb) {                                                \
+        case 11: return FN<1, 1>(__VA_ARGS__);                             \
+        case 21: return FN<2, 1>(__VA_ARGS__);                             \
+        case 31: return FN<3, 1>(__VA_ARGS__);                             \
+        case 41: return FN<4, 1>(__VA_ARGS__);                             \
+        case 12: return FN<1, 2>(__VA_ARGS__);                             \
+        case 22: return FN<2, 2>(__VA_ARGS__);                             \
+        case 42: return FN<4, 2>(__VA_ARGS__);                             \
+        default: return cudaErrorInvalidValue;                             \
+    }
+
+bool limb_gemm_supported(int na, int nb) {
+    switch (na * 10 + nb) {
+        case 11: case 21: case 31: case 41: case 12: case 22: case 42: return true;
+        default: return false;
+    }
+}
+
+int limb_gemm_rows_per_limb(int na) { return na <= 2 ? 128 : 64; }
+
+cudaError_t limb_gemm_prepare(int na, int nb) { QX_LIMB_DISPATCH(prepare_t) }
+
+cudaError_t limb_gemm_launch(int na, int nb, const MmaArgs &a, int grid, cudaStream_t stream) {
+    QX_LIMB_DISPATCH(launch_t, a, grid, stream)
+}
+
+}  // namespace qx

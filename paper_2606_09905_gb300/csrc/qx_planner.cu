@@ -1,0 +1,134 @@
+// qx_planner.cu -- operand-range contracts -> exact limb schemes (paper:
+// Methodology, "operand-range contracts propagate to higher-level operators
+// to determine feasible tiling, packing, and accumulation at runtime").
+//
+// A declared range [lo, hi] for each operand decides
+//   - packing:      how many balanced base-2^s digits each operand needs so
+//                   that every digit is an exact FP16 integer (|digit| <= 2048);
+//   - accumulation: how many K terms an FP32 accumulator may take before a
+//                   partial sum could pass 2^24 (the last integer magnitude up
+//                   to which binary32 is exact), i.e. the chunk length after
+//                   which the epilogue moves the sums into int32;
+//   - tiling:       the tile shape that follows from the digit counts (the
+//                   N-side digits are stacked along the MMA's N dimension).
+// Host code only; it runs at plan creation and in qx_plan_query.
+#include <algorithm>
+#include <cstdint>
+
+#include "qx_internal.h"
+
+namespace qx {
+
+bool limb_gemm_supported(int na, int nb);
+int limb_gemm_rows_per_limb(int na);
+
+static int64_t iabs64(int64_t v) { return v < 0 ? -v : v; }
+
+// Top digit left after `limbs - 1` balanced digit extractions of x.
+static int64_t top_digit(int64_t x, int limbs, int s) {
+    const int64_t half = int64_t(1) << (s - 1);
+    const int64_t mask = (int64_t(1) << s) - 1;
+    for (int i = 0; i < limbs - 1; ++i) {
+        const int64_t d = ((x + half) & mask) - half;
+        x = (x - d) / (int64_t(1) << s);
+    }
+    return x;
+}
+
+// Digit bounds of [lo, hi] split into `limbs` digits of `s` bits.  False if a
+// digit could leave the exact-FP16 range or the device's int32 digit
+// arithmetic could overflow.
+bool make_split(qx_range r, int limbs, int s, Split *out) {
+    Split sp;
+    sp.limbs = limbs;
+    sp.shift = limbs == 1 ? 0 : s;
+    const int64_t mag = std::max(iabs64(r.lo), iabs64(r.hi));
+    if (limbs == 1) {
+        sp.bound[0] = mag;
+    } else {
+        if (s < 1 || s > 12 || mag >= (int64_t(1) << 30)) return false;
+        for (int i = 0; i < limbs - 1; ++i) sp.bound[i] = int64_t(1) << (s - 1);
+        // the top digit is monotone in x, so its extremes sit at lo and hi
+        sp.bound[limbs - 1] = std::max(iabs64(top_digit(r.lo, limbs, s)), iabs64(top_digit(r.hi, limbs, s)));
+    }
+    for (int i = 0; i < limbs; ++i)
+        if (sp.bound[i] > kHalfExact) return false;
+    *out = sp;
+    return true;
+}
+
+static int64_t per_term_bound(const Split &n, const Split &m) {
+    int64_t worst = 0;
+    for (int i = 0; i < n.limbs; ++i)
+        for (int j = 0; j < m.limbs; ++j) worst = std::max(worst, n.bound[i] * m.bound[j]);
+    return std::max<int64_t>(worst, 1);
+}
+
+// Best scheme for a K-long contraction between an N-side operand with range
+// rn and an M-side operand with range rm.  False if no supported scheme is
+// exact.
+bool plan_contraction(qx_range rn, qx_range rm, int64_t K, Scheme *best) {
+    const int64_t kb = std::max<int64_t>(1, (K + kBK - 1) / kBK);
+    double best_cost = 0;
+    bool found = false;
+    for (int na = 1; na <= 4; ++na) {
+        for (int sa = (na == 1 ? 0 : 1); sa <= (na == 1 ? 0 : 12); ++sa) {
+            Split sn;
+            if (!make_split(rn, na, sa, &sn)) continue;
+            for (int nb = 1; nb <= 2; ++nb) {
+                for (int sb = (nb == 1 ? 0 : 1); sb <= (nb == 1 ? 0 : 12); ++sb) {
+                    if (!limb_gemm_supported(na, nb)) continue;
+                    Split sm;
+                    if (!make_split(rm, nb, sb, &sm)) continue;
+                    if ((na - 1) * sn.shift + (nb - 1) * sm.shift > 31) continue;
+                    const int64_t per = per_term_bound(sn, sm);
+                    int64_t chunk_kb = (kAccLimit / per) / kBK;
+                    if (chunk_kb < 1) continue;
+                    chunk_kb = std::min(chunk_kb, kb);
+                    const int64_t n_chunks = (kb + chunk_kb - 1) / chunk_kb;
+                    chunk_kb = (kb + n_chunks - 1) / n_chunks;  // balance the chunks
+                    const int mr = limb_gemm_rows_per_limb(na);
+                    const bool double_buffered = nb * na * mr <= 256;
+                    // Time per output element, relative units.  Per limb
+                    // pair, one k-block of MMA costs 2 and draining one
+                    // chunk's accumulators costs about 11 (FP32 -> int32
+                    // conversion runs at a fraction of the ALU rate).  With
+                    // double-buffered accumulators the drain overlaps the
+                    // next chunk's MMAs, otherwise the MMAs wait for it.
+                    const double t_mma = 2.0 * double(chunk_kb);
+                    const double t_drain = 11.0;
+                    const double per_chunk =
+                        double_buffered ? std::max(t_mma, t_drain) : t_mma + t_drain;
+                    double cost = double(na * nb) * double(n_chunks) * per_chunk;
+                    // tie-break: fewer chunks, then N-side digits (one MMA covers them)
+                    cost += 1e-3 * double(n_chunks) + 1e-6 * double(nb);
+                    if (!found || cost < best_cost) {
+                        found = true;
+                        best_cost = cost;
+                        best->n = sn;
+                        best->m = sm;
+                        best->k = K;
+                        best->chunk_kb = chunk_kb;
+                        best->n_chunks = K > 0 ? n_chunks : 0;
+                        best->acc_bound = chunk_kb * kBK * per;
+                    }
+                }
+            }
+        }
+    }
+    return found;
+}
+
+void scheme_to_info(const Scheme &s, qx_scheme_info *o) {
+    o->limbs_a = s.n.limbs;
+    o->shift_a = s.n.shift;
+    o->limbs_b = s.m.limbs;
+    o->shift_b = s.m.shift;
+    o->mma_per_kstep = s.n.limbs * s.m.limbs;
+    o->chunk_k = s.chunk_kb * kBK;
+    o->n_chunks = s.n_chunks;
+    o->acc_bound = s.acc_bound;
+    o->k = s.k;
+}
+
+}  // namespace qx

@@ -1,0 +1,396 @@
+// qx_prepass.cu -- operand packing (paper: Abstract and Table 1, "packed"
+// INT16 input; Methodology, operand-range contracts decide packing).
+//
+// Each integer operand is rewritten once per call into FP16 limb planes in
+// the plan's workspace: plane i holds the i-th balanced base-2^shift digit of
+// every element (an exact FP16 integer), laid out K-major so the TMA loads of
+// the tiled limb GEMM read 128-byte rows.  The GEMM's B is transposed on the
+// way (K x N -> N x K); the conv input goes NCHW -> NHWC with channels padded
+// to a multiple of 64 (zeros); conv weights go KCRS -> K,R,S,C.  With range
+// checking on, every operand is compared with its declared range and a
+// violation sets QX_ERR_CONTRACT in the plan's device error word.
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include "qx_device.cuh"
+#include "qx_internal.h"
+
+namespace qx {
+
+struct RangeCheck {
+    int on;
+    int64_t lo, hi;
+    __device__ __forceinline__ void test(int32_t v, int *err) const {
+        if (on && (v < lo || v > hi)) atomicCAS(err, 0, kErrContract);
+    }
+};
+
+template <int NL>
+__device__ __forceinline__ void store_limbs8(__half *plane0, int64_t plane_stride, const int32_t (&v)[8],
+                                             int shift) {
+    int32_t d[8][NL];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) split_digits<NL>(v[e], shift, d[e]);
+#pragma unroll
+    for (int i = 0; i < NL; ++i) {
+        __align__(16) __half h[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) h[e] = __int2half_rn(d[e][i]);
+        *reinterpret_cast<uint4 *>(plane0 + i * plane_stride) = *reinterpret_cast<uint4 *>(h);
+    }
+}
+
+template <typename T>
+__device__ __forceinline__ void load8(const T *src, bool vec, int valid, int32_t (&v)[8]) {
+    if (vec) {
+        if constexpr (sizeof(T) == 2) {
+            const uint4 u = __ldg(reinterpret_cast<const uint4 *>(src));
+            const int16_t *s = reinterpret_cast<const int16_t *>(&u);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = s[e];
+        } else {
+            const uint4 u0 = __ldg(reinterpret_cast<const uint4 *>(src));
+            const uint4 u1 = __ldg(reinterpret_cast<const uint4 *>(src) + 1);
+            const int32_t *s0 = reinterpret_cast<const int32_t *>(&u0);
+            const int32_t *s1 = reinterpret_cast<const int32_t *>(&u1);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                v[e] = s0[e];
+                v[e + 4] = s1[e];
+            }
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = e < valid ? int32_t(src[e]) : 0;
+    }
+}
+
+// ------------------------------------------------------------ GEMM operands
+struct GemmPackArgs {
+    const void *A, *B;
+    int64_t lda, ldb;
+    int M, N, K, Kp;
+    __half *a_planes;      // na planes of M x Kp
+    __half *bt_planes;     // nb planes of N x Kp
+    int shift_a, shift_b;
+    RangeCheck ca, cb;
+    int *err;
+    int a_blocks;          // blocks [0, a_blocks) pack A, the rest transpose B
+    int b_tiles_n;         // B tiles along N (64 wide)
+    int vec_a;             // A rows 16-byte aligned for 8-element loads
+};
+
+template <typename T, int NA, int NB>
+__global__ void __launch_bounds__(256) pack_gemm_kernel(const GemmPackArgs p) {
+    __shared__ int32_t tile[64][65];
+    const T *A = static_cast<const T *>(p.A);
+    const T *B = static_cast<const T *>(p.B);
+    if (int(blockIdx.x) < p.a_blocks) {
+        // A (M x K, row-major) -> NA planes of M x Kp, 8 consecutive k per thread
+        const int kg_per_row = (p.K + 7) >> 3;
+        const int64_t items = int64_t(p.M) * kg_per_row;
+        const int64_t plane_stride = int64_t(p.M) * p.Kp;
+        for (int64_t it = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; it < items;
+             it += int64_t(p.a_blocks) * blockDim.x) {
+            const int row = int(it / kg_per_row);
+            const int k = int(it - int64_t(row) * kg_per_row) * 8;
+            const int valid = min(8, p.K - k);
+            int32_t v[8];
+            load8<T>(A + int64_t(row) * p.lda + k, p.vec_a && valid == 8, valid, v);
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                if (e < valid) p.ca.test(v[e], p.err);
+            store_limbs8<NA>(p.a_planes + int64_t(row) * p.Kp + k, plane_stride, v, p.shift_a);
+        }
+        return;
+    }
+    // B (K x N, row-major) -> NB planes of N x Kp: 64 x 64 tiles through smem
+    const int t = int(blockIdx.x) - p.a_blocks;
+    const int n0 = (t % p.b_tiles_n) * 64;
+    const int k0 = (t / p.b_tiles_n) * 64;
+    for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
+        const int kr = i >> 6, nc = i & 63;
+        int32_t v = 0;
+        if (k0 + kr < p.K && n0 + nc < p.N) {
+            v = int32_t(B[int64_t(k0 + kr) * p.ldb + n0 + nc]);
+            p.cb.test(v, p.err);
+        }
+        tile[kr][nc] = v;
+    }
+    __syncthreads();
+    const int64_t plane_stride = int64_t(p.N) * p.Kp;
+    for (int i = threadIdx.x; i < 64 * 8; i += blockDim.x) {
+        const int nr = i >> 3, kg = i & 7;
+        const int n = n0 + nr, k = k0 + kg * 8;
+        if (n >= p.N || k >= p.Kp) continue;
+        int32_t v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = tile[kg * 8 + e][nr];
+        store_limbs8<NB>(p.bt_planes + int64_t(n) * p.Kp + k, plane_stride, v, p.shift_b);
+    }
+}
+
+// ------------------------------------------------------------ conv operands
+struct ConvPackArgs {
+    const void *x, *w;
+    int n, c, h, wd, k_out, r, s, Cp;
+    __half *x_planes;      // nx planes of n x h x w x Cp
+    __half *w_planes;      // nw planes of k_out x r x s x Cp
+    int shift_x, shift_w;
+    RangeCheck cx, cw;
+    int *err;
+    int x_blocks;          // blocks [0, x_blocks) transpose x; the rest pack w
+    int x_tiles_hw, x_tiles_c;
+};
+
+template <typename T, int NX, int NW>
+__global__ void __launch_bounds__(256) pack_conv_kernel(const ConvPackArgs p) {
+    __shared__ int32_t tile[64][65];
+    const T *X = static_cast<const T *>(p.x);
+    const T *W = static_cast<const T *>(p.w);
+    const int HW = p.h * p.wd;
+    if (int(blockIdx.x) < p.x_blocks) {
+        // one 64 (channels) x 64 (pixels) tile of one image: NCHW -> NHWC
+        int t = blockIdx.x;
+        const int tc = t % p.x_tiles_c;
+        t /= p.x_tiles_c;
+        const int thw = t % p.x_tiles_hw;
+        const int img = t / p.x_tiles_hw;
+        const int c0 = tc * 64, hw0 = thw * 64;
+        for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
+            const int cr = i >> 6, pc = i & 63;
+            int32_t v = 0;
+            if (c0 + cr < p.c && hw0 + pc < HW) {
+                v = int32_t(X[(int64_t(img) * p.c + c0 + cr) * HW + hw0 + pc]);
+                p.cx.test(v, p.err);
+            }
+            tile[cr][pc] = v;
+        }
+        __syncthreads();
+        const int64_t plane_stride = int64_t(p.n) * HW * p.Cp;
+        for (int i = threadIdx.x; i < 64 * 8; i += blockDim.x) {
+            const int pr = i >> 3, cg = i & 7;
+            if (hw0 + pr >= HW) continue;
+            int32_t v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = tile[cg * 8 + e][pr];
+            store_limbs8<NX>(p.x_planes + (int64_t(img) * HW + hw0 + pr) * p.Cp + c0 + cg * 8,
+                             plane_stride, v, p.shift_x);
+        }
+        return;
+    }
+    // weights: KCRS -> (k, r, s, Cp), 8 channels per thread
+    const int RS = p.r * p.s;
+    const int cgs = p.Cp >> 3;
+    const int64_t items = int64_t(p.k_out) * RS * cgs;
+    const int64_t plane_stride = int64_t(p.k_out) * RS * p.Cp;
+    for (int64_t it = int64_t(blockIdx.x - p.x_blocks) * blockDim.x + threadIdx.x; it < items;
+         it += int64_t(gridDim.x - p.x_blocks) * blockDim.x) {
+        const int cg = int(it % cgs);
+        const int tap = int((it / cgs) % RS);
+        const int o = int(it / (int64_t(cgs) * RS));
+        int32_t v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int c = cg * 8 + e;
+            v[e] = 0;
+            if (c < p.c) {
+                v[e] = int32_t(W[(int64_t(o) * p.c + c) * RS + tap]);
+                p.cw.test(v[e], p.err);
+            }
+        }
+        store_limbs8<NW>(p.w_planes + (int64_t(o) * RS + tap) * p.Cp + cg * 8, plane_stride, v,
+                         p.shift_w);
+    }
+}
+
+// ------------------------------------------------------- attention operands
+struct AttnPackArgs {
+    const void *Q, *K, *V;
+    int L, d, dp, Lp;
+    __half *q, *k;          // L x dp each
+    __half *vt;             // dp x Lp (V transposed, keys contiguous)
+    RangeCheck cq, ck, cv;
+    int *err;
+    int qk_blocks;          // blocks [0, qk_blocks) pack Q and K; the rest transpose V
+    int v_tiles_l;
+};
+
+template <typename T>
+__global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
+    __shared__ int32_t tile[64][65];
+    const T *Q = static_cast<const T *>(p.Q);
+    const T *K = static_cast<const T *>(p.K);
+    const T *V = static_cast<const T *>(p.V);
+    if (int(blockIdx.x) < p.qk_blocks) {
+        const int gpr = p.dp >> 3;
+        const int64_t items = int64_t(2) * p.L * gpr;
+        for (int64_t it = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; it < items;
+             it += int64_t(p.qk_blocks) * blockDim.x) {
+            const int which = int(it / (int64_t(p.L) * gpr));
+            const int64_t rem = it - int64_t(which) * p.L * gpr;
+            const int row = int(rem / gpr);
+            const int c = int(rem - int64_t(row) * gpr) * 8;
+            const T *src = (which ? K : Q) + int64_t(row) * p.d;
+            const RangeCheck &ch = which ? p.ck : p.cq;
+            int32_t v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                v[e] = 0;
+                if (c + e < p.d) {
+                    v[e] = int32_t(src[c + e]);
+                    ch.test(v[e], p.err);
+                }
+            }
+            store_limbs8<1>((which ? p.k : p.q) + int64_t(row) * p.dp + c, 0, v, 0);
+        }
+        return;
+    }
+    const int t = int(blockIdx.x) - p.qk_blocks;
+    const int l0 = (t % p.v_tiles_l) * 64;
+    const int c0 = (t / p.v_tiles_l) * 64;
+    for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
+        const int lr = i >> 6, cc = i & 63;
+        int32_t v = 0;
+        if (l0 + lr < p.L && c0 + cc < p.d) {
+            v = int32_t(V[int64_t(l0 + lr) * p.d + c0 + cc]);
+            p.cv.test(v, p.err);
+        }
+        tile[lr][cc] = v;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < 64 * 8; i += blockDim.x) {
+        const int cr = i >> 3, lg = i & 7;
+        const int c = c0 + cr, l = l0 + lg * 8;
+        if (c >= p.dp || l >= p.Lp) continue;
+        int32_t v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = tile[lg * 8 + e][cr];
+        store_limbs8<1>(p.vt + int64_t(c) * p.Lp + l, 0, v, 0);
+    }
+}
+
+// ------------------------------------------------------------------- host
+static RangeCheck make_check(int on, qx_range r) { return RangeCheck{on, r.lo, r.hi}; }
+
+template <typename T>
+static cudaError_t pack_gemm_t(int na, int nb, const GemmPackArgs &p, int grid, cudaStream_t st) {
+#define QX_PG(A_, B_)                                                                  \
+    if (na == A_ && nb == B_) {                                                        \
+        pack_gemm_kernel<T, A_, B_><<<grid, 256, 0, st>>>(p);                          \
+        return cudaGetLastError();                                                     \
+    }
+    QX_PG(1, 1) QX_PG(2, 1) QX_PG(3, 1) QX_PG(4, 1) QX_PG(1, 2) QX_PG(2, 2) QX_PG(4, 2)
+#undef QX_PG
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_pack_gemm(bool i32, const void *A, const void *B, int64_t lda, int64_t ldb,
+                             int M, int N, int K, int Kp, __half *a_planes, __half *bt_planes,
+                             int na, int shift_a, int nb, int shift_b, int check, qx_range ra,
+                             qx_range rb, int *err, int num_sms, cudaStream_t st) {
+    GemmPackArgs p;
+    p.A = A;
+    p.B = B;
+    p.lda = lda;
+    p.ldb = ldb;
+    p.M = M;
+    p.N = N;
+    p.K = K;
+    p.Kp = Kp;
+    p.a_planes = a_planes;
+    p.bt_planes = bt_planes;
+    p.shift_a = shift_a;
+    p.shift_b = shift_b;
+    p.ca = make_check(check, ra);
+    p.cb = make_check(check, rb);
+    p.err = err;
+    const int esz = i32 ? 4 : 2;
+    p.vec_a = (reinterpret_cast<uintptr_t>(A) % 16 == 0) && ((lda * esz) % 16 == 0);
+    const int64_t a_items = int64_t(M) * ((K + 7) / 8);
+    const int64_t a_blocks = (a_items + 255) / 256;
+    p.a_blocks = int(a_blocks < int64_t(num_sms) * 8 ? a_blocks : int64_t(num_sms) * 8);
+    p.b_tiles_n = (N + 63) / 64;
+    const int64_t b_blocks = int64_t(p.b_tiles_n) * ((K + 63) / 64);
+    const int64_t grid = p.a_blocks + b_blocks;
+    if (grid <= 0) return cudaSuccess;
+    return i32 ? pack_gemm_t<int32_t>(na, nb, p, int(grid), st)
+               : pack_gemm_t<int16_t>(na, nb, p, int(grid), st);
+}
+
+template <typename T>
+static cudaError_t pack_conv_t(int nx, int nw, const ConvPackArgs &p, int grid, cudaStream_t st) {
+#define QX_PC(A_, B_)                                                                  \
+    if (nx == A_ && nw == B_) {                                                        \
+        pack_conv_kernel<T, A_, B_><<<grid, 256, 0, st>>>(p);                          \
+        return cudaGetLastError();                                                     \
+    }
+    QX_PC(1, 1) QX_PC(1, 2) QX_PC(1, 3) QX_PC(1, 4) QX_PC(2, 1) QX_PC(2, 2) QX_PC(2, 4)
+#undef QX_PC
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_pack_conv(bool i32, const void *x, const void *w, int n, int c, int h, int wd,
+                             int k_out, int r, int s, int Cp, __half *x_planes, __half *w_planes,
+                             int nx, int shift_x, int nw, int shift_w, int check, qx_range rx,
+                             qx_range rw, int *err, int num_sms, cudaStream_t st) {
+    ConvPackArgs p;
+    p.x = x;
+    p.w = w;
+    p.n = n;
+    p.c = c;
+    p.h = h;
+    p.wd = wd;
+    p.k_out = k_out;
+    p.r = r;
+    p.s = s;
+    p.Cp = Cp;
+    p.x_planes = x_planes;
+    p.w_planes = w_planes;
+    p.shift_x = shift_x;
+    p.shift_w = shift_w;
+    p.cx = make_check(check, rx);
+    p.cw = make_check(check, rw);
+    p.err = err;
+    p.x_tiles_hw = (h * wd + 63) / 64;
+    p.x_tiles_c = Cp / 64;
+    p.x_blocks = n * p.x_tiles_hw * p.x_tiles_c;
+    const int64_t w_items = int64_t(k_out) * r * s * (Cp / 8);
+    int w_blocks = int((w_items + 255) / 256);
+    if (w_blocks > num_sms) w_blocks = num_sms;
+    if (w_blocks < 1) w_blocks = 1;
+    const int grid = p.x_blocks + w_blocks;
+    return i32 ? pack_conv_t<int32_t>(nx, nw, p, grid, st) : pack_conv_t<int16_t>(nx, nw, p, grid, st);
+}
+
+cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int L, int d,
+                             int dp, int Lp, __half *q, __half *k, __half *vt, int check,
+                             qx_range rq, qx_range rk, qx_range rv, int *err, int num_sms,
+                             cudaStream_t st) {
+    AttnPackArgs p;
+    p.Q = Q;
+    p.K = K;
+    p.V = V;
+    p.L = L;
+    p.d = d;
+    p.dp = dp;
+    p.Lp = Lp;
+    p.q = q;
+    p.k = k;
+    p.vt = vt;
+    p.cq = make_check(check, rq);
+    p.ck = make_check(check, rk);
+    p.cv = make_check(check, rv);
+    p.err = err;
+    const int64_t qk_items = int64_t(2) * L * (dp / 8);
+    int64_t qk_blocks = (qk_items + 255) / 256;
+    if (qk_blocks > num_sms) qk_blocks = num_sms;
+    p.qk_blocks = int(qk_blocks);
+    p.v_tiles_l = (Lp + 63) / 64;
+    const int grid = p.qk_blocks + p.v_tiles_l * ((dp + 63) / 64);
+    if (i32) pack_attn_kernel<int32_t><<<grid, 256, 0, st>>>(p);
+    else pack_attn_kernel<int16_t><<<grid, 256, 0, st>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace qx

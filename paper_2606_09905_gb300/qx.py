@@ -1,0 +1,255 @@
+"""ctypes binding over the C ABI of libqx.so (include/qx.h).
+
+Argument marshalling only: every step of the computation runs in the CUDA
+library.  PyTorch supplies device memory and streams; tensors are passed as
+raw device pointers on the current CUDA stream.  If the library is missing
+the binding raises -- there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from dataclasses import dataclass
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libqx.so")
+
+# qx_status
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CONTRACT, ERR_OOM, ERR_CUDA, ERR_TIMEOUT, ERR_DEVICE = range(8)
+# qx_op / qx_dtype
+OP_GEMM, OP_CONV2D, OP_ATTN = 0, 1, 2
+I16, I32, F32 = 0, 1, 2
+FLAG_CHECK_RANGES = 1
+
+# Every function the header declares; the CPU tests check the exports.
+EXPORTS = ("qx_plan_create", "qx_plan_destroy", "qx_plan_query", "qx_plan_info",
+           "qx_gemm_i16_i32", "qx_gemm_i32", "qx_conv2d_gemm", "qx_attn_core",
+           "qx_plan_status", "qx_status_string", "qx_last_error", "qx_version")
+
+
+class QxError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str):
+        self.status = status
+        super().__init__(f"{where}: {detail} (status {status})")
+
+
+class Range(ctypes.Structure):
+    _fields_ = [("lo", ctypes.c_int64), ("hi", ctypes.c_int64)]
+
+
+class PlanDesc(ctypes.Structure):
+    _fields_ = [("op", ctypes.c_int), ("in_dtype", ctypes.c_int),
+                ("M", ctypes.c_int64), ("N", ctypes.c_int64), ("K", ctypes.c_int64),
+                ("lda", ctypes.c_int64), ("ldb", ctypes.c_int64), ("ldc", ctypes.c_int64),
+                ("n", ctypes.c_int64), ("c", ctypes.c_int64), ("h", ctypes.c_int64),
+                ("w", ctypes.c_int64), ("k_out", ctypes.c_int64), ("r", ctypes.c_int64),
+                ("s", ctypes.c_int64), ("stride", ctypes.c_int64), ("pad", ctypes.c_int64),
+                ("L", ctypes.c_int64), ("d", ctypes.c_int64),
+                ("range_a", Range), ("range_b", Range), ("range_c", Range),
+                ("flags", ctypes.c_uint)]
+
+
+class SchemeInfo(ctypes.Structure):
+    _fields_ = [("limbs_a", ctypes.c_int), ("shift_a", ctypes.c_int),
+                ("limbs_b", ctypes.c_int), ("shift_b", ctypes.c_int),
+                ("mma_per_kstep", ctypes.c_int),
+                ("chunk_k", ctypes.c_int64), ("n_chunks", ctypes.c_int64),
+                ("acc_bound", ctypes.c_int64), ("k", ctypes.c_int64)]
+
+    def as_dict(self) -> dict:
+        return {f: getattr(self, f) for f, _ in self._fields_}
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def load() -> ctypes.CDLL:
+    """Open libqx.so (built by __graft_entry__.build()); raise if absent."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is not built; run __graft_entry__.build() first")
+        lib = ctypes.CDLL(LIB_PATH)
+        P, V = ctypes.c_void_p, ctypes.c_void_p
+        sig = {
+            "qx_plan_create": ([ctypes.POINTER(PlanDesc), ctypes.c_int, ctypes.POINTER(P)], ctypes.c_int),
+            "qx_plan_destroy": ([P], ctypes.c_int),
+            "qx_plan_query": ([ctypes.POINTER(PlanDesc), ctypes.POINTER(SchemeInfo),
+                               ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
+            "qx_plan_info": ([P, ctypes.POINTER(SchemeInfo), ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
+            "qx_gemm_i16_i32": ([P, V, V, V, V], ctypes.c_int),
+            "qx_gemm_i32": ([P, V, V, V, V], ctypes.c_int),
+            "qx_conv2d_gemm": ([P, V, V, V, V], ctypes.c_int),
+            "qx_attn_core": ([P, V, V, V, V, V], ctypes.c_int),
+            "qx_plan_status": ([P], ctypes.c_int),
+            "qx_status_string": ([ctypes.c_int], ctypes.c_char_p),
+            "qx_last_error": ([], ctypes.c_char_p),
+            "qx_version": ([], ctypes.c_int),
+        }
+        for name, (args, res) in sig.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = lib
+        return lib
+
+
+def _check(status: int, where: str):
+    if status != OK:
+        lib = load()
+        raise QxError(status, where, lib.qx_last_error().decode() or
+                      lib.qx_status_string(status).decode())
+
+
+# ------------------------------------------------------------ descriptors
+def _rng(r) -> Range:
+    return Range(int(r[0]), int(r[1]))
+
+
+def gemm_desc(M, N, K, range_a, range_b, dtype=I16, lda=0, ldb=0, ldc=0, flags=0) -> PlanDesc:
+    return PlanDesc(op=OP_GEMM, in_dtype=dtype, M=M, N=N, K=K, lda=lda, ldb=ldb, ldc=ldc,
+                    range_a=_rng(range_a), range_b=_rng(range_b), flags=flags)
+
+
+def conv_desc(n, c, h, w, k_out, r, s, stride, pad, range_x, range_w, dtype=I16, flags=0) -> PlanDesc:
+    return PlanDesc(op=OP_CONV2D, in_dtype=dtype, n=n, c=c, h=h, w=w, k_out=k_out, r=r, s=s,
+                    stride=stride, pad=pad, range_a=_rng(range_x), range_b=_rng(range_w),
+                    flags=flags)
+
+
+def attn_desc(L, d, range_q, range_k, range_v, dtype=I16, flags=0) -> PlanDesc:
+    return PlanDesc(op=OP_ATTN, in_dtype=dtype, L=L, d=d, range_a=_rng(range_q),
+                    range_b=_rng(range_k), range_c=_rng(range_v), flags=flags)
+
+
+def query(desc: PlanDesc) -> list[dict]:
+    """Host-only planner: the exact limb scheme(s) for a descriptor."""
+    lib = load()
+    out = (SchemeInfo * 2)()
+    n = ctypes.c_int(0)
+    _check(lib.qx_plan_query(ctypes.byref(desc), out, ctypes.byref(n)), "qx_plan_query")
+    return [out[i].as_dict() for i in range(n.value)]
+
+
+# ------------------------------------------------------------------- plans
+_TORCH_DT = {I16: torch.int16, I32: torch.int32, F32: torch.float32}
+
+
+def _ptr(t: torch.Tensor, dtype: torch.dtype, shape, name: str) -> int:
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+class Plan:
+    """A persistent executor: shapes, dtypes and the range contract fixed once."""
+
+    def __init__(self, desc: PlanDesc, device: int | None = None):
+        lib = load()
+        if device is None:
+            device = torch.cuda.current_device()
+        self.device = int(device)
+        self.desc = desc
+        h = ctypes.c_void_p()
+        _check(lib.qx_plan_create(ctypes.byref(desc), self.device, ctypes.byref(h)),
+               "qx_plan_create")
+        self._h = h
+
+    @property
+    def handle(self) -> ctypes.c_void_p:
+        if self._h is None:
+            raise RuntimeError("plan destroyed")
+        return self._h
+
+    def close(self):
+        if getattr(self, "_h", None) is not None:
+            _check(load().qx_plan_destroy(self._h), "qx_plan_destroy")
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def info(self) -> list[dict]:
+        out = (SchemeInfo * 2)()
+        n = ctypes.c_int(0)
+        _check(load().qx_plan_info(self.handle, out, ctypes.byref(n)), "qx_plan_info")
+        return [out[i].as_dict() for i in range(n.value)]
+
+    def status(self) -> int:
+        """Synchronise and return (and clear) the device error word as a status."""
+        return int(load().qx_plan_status(self.handle))
+
+    # -- GEMM ------------------------------------------------------------
+    def _gemm(self, fn, A, B, C, stream, dt):
+        d = self.desc
+        lda = d.lda or d.K
+        ldb = d.ldb or d.N
+        ldc = d.ldc or d.N
+        if C is None:
+            C = torch.empty((d.M, ldc), dtype=torch.int32, device=A.device)
+        a = _ptr(A, dt, (d.M, lda), "A")
+        b = _ptr(B, dt, (d.K, ldb), "B")
+        c = _ptr(C, torch.int32, (d.M, ldc), "C")
+        _check(fn(self.handle, a, b, c, _stream(stream)), fn.__name__)
+        return C
+
+    def gemm_i16_i32(self, A, B, C=None, stream=None):
+        return self._gemm(load().qx_gemm_i16_i32, A, B, C, stream, torch.int16)
+
+    def gemm_i32(self, A, B, C=None, stream=None):
+        return self._gemm(load().qx_gemm_i32, A, B, C, stream, torch.int32)
+
+    # -- conv -------------------------------------------------------------
+    def conv2d(self, x, w, y=None, stream=None):
+        d = self.desc
+        P = (d.h + 2 * d.pad - d.r) // d.stride + 1
+        Q = (d.w + 2 * d.pad - d.s) // d.stride + 1
+        dt = _TORCH_DT[d.in_dtype]
+        out_dt = torch.float32 if d.in_dtype == F32 else torch.int32
+        if y is None:
+            y = torch.empty((d.n, d.k_out, P, Q), dtype=out_dt, device=x.device)
+        px = _ptr(x, dt, (d.n, d.c, d.h, d.w), "x")
+        pw = _ptr(w, dt, (d.k_out, d.c, d.r, d.s), "w")
+        py = _ptr(y, out_dt, (d.n, d.k_out, P, Q), "y")
+        _check(load().qx_conv2d_gemm(self.handle, px, pw, py, _stream(stream)), "qx_conv2d_gemm")
+        return y
+
+    # -- attention ----------------------------------------------------------
+    def attn(self, Q, K, V, O=None, stream=None):
+        d = self.desc
+        dt = _TORCH_DT[d.in_dtype]
+        out_dt = torch.float32 if d.in_dtype == F32 else torch.int32
+        if O is None:
+            O = torch.empty((d.L, d.d), dtype=out_dt, device=Q.device)
+        shape = (d.L, d.d)
+        pq, pk, pv = (_ptr(t, dt, shape, n) for t, n in ((Q, "Q"), (K, "K"), (V, "V")))
+        po = _ptr(O, out_dt, shape, "O")
+        _check(load().qx_attn_core(self.handle, pq, pk, pv, po, _stream(stream)), "qx_attn_core")
+        return O

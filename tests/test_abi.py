@@ -1,0 +1,83 @@
+"""The C ABI library: it loads, exports every declared entry point, and its
+host-only paths (status strings, planner, argument checks) behave without a
+GPU.  No compute call is made here."""
+import ctypes
+import os
+import re
+
+import pytest
+import torch
+
+from paper_2606_09905_gb300 import qx
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "qx.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2606_09905_gb300 import _build
+    _build.build()
+    return qx.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(qx_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    assert len(names) >= 12
+    for name in names:
+        assert hasattr(lib, name), name
+    assert sorted(names) == sorted(qx.EXPORTS)
+
+
+def test_version_and_strings(lib):
+    assert lib.qx_version() == 1
+    assert lib.qx_status_string(qx.OK) == b"ok"
+    assert lib.qx_status_string(qx.ERR_CONTRACT) == b"operand-range contract"
+    assert lib.qx_status_string(99) == b"unknown status"
+
+
+def test_struct_layouts_match_header():
+    # qx_plan_desc: 2 ints, 17 int64, 3 ranges (2 x int64), 1 unsigned (+pad)
+    assert ctypes.sizeof(qx.PlanDesc) == 8 + 17 * 8 + 3 * 16 + 8
+    assert ctypes.sizeof(qx.SchemeInfo) == 5 * 4 + 4 + 4 * 8
+
+
+def test_query_workload_schemes(lib):
+    s = qx.query(qx.gemm_desc(256, 256, 256, (-1023, 1023), (-1023, 1023)))
+    assert len(s) == 1 and s[0]["mma_per_kstep"] == 2 and s[0]["n_chunks"] == 1
+    s = qx.query(qx.gemm_desc(8192, 8192, 8192, (-500, 500), (-500, 500)))[0]
+    assert s["mma_per_kstep"] == 2 and s["n_chunks"] == 4
+    s = qx.query(qx.conv_desc(8, 64, 56, 56, 128, 3, 3, 1, 1, (-255, 255), (-255, 255)))[0]
+    assert s["mma_per_kstep"] == 1 and s["n_chunks"] == 3
+    s = qx.query(qx.attn_desc(1024, 64, (-7, 7), (-7, 7), (-7, 7)))
+    assert len(s) == 2 and s[0]["acc_bound"] == 64 * 49 and s[1]["limbs_a"] == 2
+
+
+def test_query_rejects(lib):
+    with pytest.raises(qx.QxError) as e:
+        qx.query(qx.gemm_desc(4, 4, 4, (5, 1), (0, 1)))
+    assert e.value.status == qx.ERR_INVALID_ARG
+    with pytest.raises(qx.QxError) as e:
+        qx.query(qx.gemm_desc(4, 4, 4, (-40000, 1), (0, 1)))      # outside int16
+    assert e.value.status == qx.ERR_INVALID_ARG
+    with pytest.raises(qx.QxError) as e:
+        qx.query(qx.gemm_desc(-1, 4, 4, (0, 1), (0, 1)))
+    assert e.value.status == qx.ERR_INVALID_ARG
+    with pytest.raises(qx.QxError) as e:                            # needs > 2x2 limbs
+        qx.query(qx.gemm_desc(4, 4, 4, (-2**29, 2**29), (-2**29, 2**29), dtype=qx.I32))
+    assert e.value.status == qx.ERR_CONTRACT
+    with pytest.raises(qx.QxError) as e:
+        qx.query(qx.attn_desc(64, 64, (-4096, 4096), (-7, 7), (-7, 7)))
+    assert e.value.status == qx.ERR_CONTRACT
+
+
+@pytest.mark.skipif(torch.cuda.is_available(), reason="checks the no-device path")
+def test_plan_create_without_device_fails_cleanly(lib):
+    with pytest.raises(qx.QxError) as e:
+        qx.Plan(qx.gemm_desc(8, 8, 8, (-1, 1), (-1, 1)), device=0)
+    assert e.value.status in (qx.ERR_DEVICE, qx.ERR_CUDA)

@@ -1,0 +1,98 @@
+"""GPU parity of the GEMM-backed Conv2D (Table 2 Conv2D rows; lowering done on
+load by TMA im2col) against the CPU oracle's direct convolution, bit for bit."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_09905_gb300 import inputs, qx
+
+from gpu_util import assert_exact, build_once, wrap32
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    build_once()
+
+
+def conv_gpu(x, w, stride, pad, rx, rw, dtype=qx.I16, flags=0):
+    n, c, h, wd = x.shape
+    k, _, r, s = w.shape
+    with qx.Plan(qx.conv_desc(n, c, h, wd, k, r, s, stride, pad, rx, rw, dtype=dtype,
+                              flags=flags)) as plan:
+        y = plan.conv2d(x.cuda(), w.cuda())
+        torch.cuda.synchronize()
+        st = plan.status()
+        info = plan.info()
+    return y.cpu().numpy().astype(np.int64), st, info
+
+
+def test_conv_workload_int16():
+    """8 x 64 x 56 x 56 input, 128 x 64 x 3 x 3 weights, stride 1, pad 1."""
+    x, w = inputs.conv_case(8, 64, 56, 56, 128, 3, 3, -255, 255, seed=0)
+    ref = oracle.conv2d(x, w, 1, 1)
+    got, st, info = conv_gpu(x, w, 1, 1, (-255, 255), (-255, 255))
+    assert st == qx.OK
+    assert_exact(got, ref, f"conv workload {info}")
+
+
+def test_conv_workload_int32():
+    x, w = inputs.conv_case(8, 64, 56, 56, 128, 3, 3, -255, 255, seed=1, dtype=torch.int32)
+    ref = oracle.conv2d(x, w, 1, 1)
+    got, st, _ = conv_gpu(x, w, 1, 1, (-255, 255), (-255, 255), dtype=qx.I32)
+    assert st == qx.OK
+    assert_exact(got, ref, "conv int32")
+
+
+@pytest.mark.parametrize("shape,stride,pad", [
+    ((1, 3, 7, 9, 5, 3, 3), 1, 1),
+    ((2, 64, 16, 16, 64, 3, 3), 1, 1),
+    ((3, 130, 9, 11, 200, 3, 3), 1, 1),
+    ((2, 16, 12, 10, 24, 1, 1), 1, 0),
+    ((1, 8, 13, 12, 16, 5, 3), 1, 2),
+    ((2, 32, 15, 15, 40, 3, 3), 1, 0),
+    ((1, 64, 30, 30, 64, 3, 3), 2, 1),
+    ((2, 16, 17, 13, 32, 3, 3), 2, 0),
+])
+def test_conv_shapes(shape, stride, pad):
+    n, c, h, wd, k, r, s = shape
+    x, w = inputs.conv_case(n, c, h, wd, k, r, s, -255, 255, seed=sum(shape) + stride)
+    ref = oracle.conv2d(x, w, stride, pad)
+    got, st, info = conv_gpu(x, w, stride, pad, (-255, 255), (-255, 255))
+    assert st == qx.OK
+    assert_exact(got, ref, f"conv {shape} stride {stride} pad {pad} {info}")
+
+
+def test_conv_all_ones_borders():
+    x = torch.ones((1, 64, 8, 8), dtype=torch.int16)
+    w = torch.ones((64, 64, 3, 3), dtype=torch.int16)
+    got, st, _ = conv_gpu(x, w, 1, 1, (0, 1), (0, 1))
+    assert st == qx.OK
+    exp = np.full((8, 8), 9 * 64)
+    exp[0, :] = exp[-1, :] = exp[:, 0] = exp[:, -1] = 6 * 64
+    exp[0, 0] = exp[0, -1] = exp[-1, 0] = exp[-1, -1] = 4 * 64
+    assert (got[0] == exp).all()
+
+
+@pytest.mark.parametrize("rx,rw", [((-20000, 20000), (-255, 255)),
+                                   ((-255, 255), (-30000, 30000)),
+                                   ((-2**20, 2**20), (-2**11, 2**11))])
+def test_conv_limb_schemes_int32(rx, rw):
+    n, c, h, wd, k, r, s = 2, 16, 9, 9, 24, 3, 3
+    g = torch.Generator().manual_seed(rx[1] % 1000)
+    x = torch.randint(rx[0], rx[1] + 1, (n, c, h, wd), generator=g, dtype=torch.int32)
+    w = torch.randint(rw[0], rw[1] + 1, (k, c, r, s), generator=g, dtype=torch.int32)
+    ref = oracle.conv2d(x, w, 1, 1)
+    got, st, info = conv_gpu(x, w, 1, 1, rx, rw, dtype=qx.I32)
+    assert st == qx.OK
+    assert info[0]["mma_per_kstep"] > 1
+    assert_exact(got, wrap32(ref), f"conv limbs {info}")
+
+
+def test_conv_range_check():
+    x, w = inputs.conv_case(1, 8, 6, 6, 8, 3, 3, -10, 10, seed=2)
+    w[3, 2, 1, 1] = -11
+    _, st, _ = conv_gpu(x, w, 1, 1, (-10, 10), (-10, 10), flags=qx.FLAG_CHECK_RANGES)
+    assert st == qx.ERR_CONTRACT
