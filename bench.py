@@ -1,0 +1,466 @@
+#!/usr/bin/env python3
+"""Benchmark of the exact integer GEMM substrate on GB300.
+
+Step = one execution of the hot path on the 8192^3 INT16 workload (values
+uniform in [-500, 500]): operand packing into FP16 limb planes, then the
+tcgen05 limb GEMM with int32 recombination -- i.e. one qx_gemm_i16_i32 call
+(issued as its two halves, qx_pack and qx_run_packed, so the tensor-core
+kernel can be timed by itself).  Inputs are resident in HBM; A and B (128 MiB
+each), their limb planes (384 MiB) and C (256 MiB) all exceed the 129 MB L2,
+so no flush is needed between steps.
+
+Prints one JSON line (rank 0).  `value` is whole-job TOPS (2*M*N*K integer
+ops per step, summed over ranks: each rank runs its own problem, weak
+scaling).  Extra keys: `e2e` (same metric through the public API with pinned
+host buffers, copies inside the timed region), `roofline` (the limb GEMM
+kernel against the measured dense FP16/BF16 tensor peak), `cpu_baseline`
+(the CPU oracle on a row sample), `clocks` (nvidia-smi during the timed
+region), `operators` (setup / cached steady-state / execute-only times and
+GOPS of the GEMM, the Conv2D and the attention workloads, as the paper
+reports them).
+
+`--impl reference` times the CPU oracle (the only reference for this path)
+on the host cores instead, same metric and unit.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "INT16-in/INT32-acc GEMM TOPS at 8192^3; conv/attn GOPS; % of roofline"
+M = N = K = 8192
+LO, HI = -500, 500
+
+
+def workload_name():
+    return (f"gemm{M}: INT16-in/INT32-acc GEMM C=A*B, M=N=K={M}, row-major, "
+            f"values i.i.d. uniform [{LO},{HI}]")
+
+
+def _env_int(name, default):
+    try:
+        return int(os.environ.get(name, default))
+    except ValueError:
+        return default
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons while running."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="qx_clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", self.gpu_id],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+
+        def num(v):
+            try:
+                return float(v)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        power = [num(r[3]) for r in rows if num(r[3]) is not None]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": max(power) if power else None}
+
+
+def gpu_smi_id(torch, dev_index):
+    try:
+        props = torch.cuda.get_device_properties(dev_index)
+        bus = getattr(props, "pci_bus_id", None)
+        dom = getattr(props, "pci_domain_id", None)
+        devid = getattr(props, "pci_device_id", None)
+        if bus is not None and dom is not None and devid is not None:
+            return f"{dom:08x}:{bus:02x}:{devid:02x}.0"
+    except Exception:
+        pass
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [v.strip() for v in vis.split(",") if v.strip()]
+        if dev_index < len(ids):
+            return ids[dev_index]
+    return str(dev_index)
+
+
+# ------------------------------------------------------------ CPU baseline
+def cpu_oracle_gemm(rows: int, seed: int = 0):
+    """The CPU oracle (plain C, int64 accumulation) computing `rows` rows of
+    the 8192^3 product.  Returns (seconds, threads)."""
+    import oracle
+    from paper_2606_09905_gb300 import inputs
+    A, B = inputs.gemm_case(M, N, K, LO, HI, seed)
+    a = A[:rows].numpy()
+    b = B.numpy()
+    oracle.gemm(a[:1], b)            # load and warm the library
+    t0 = time.perf_counter()
+    oracle.gemm(a, b)
+    return time.perf_counter() - t0, oracle.threads()
+
+
+def calibrate_rows(target_s: float) -> int:
+    import oracle
+    probe = max(16, 2 * oracle.threads())      # enough rows to occupy every thread
+    t, _ = cpu_oracle_gemm(probe)
+    per_row = max(t / probe, 1e-5)
+    return int(max(probe, min(M, target_s / per_row)))
+
+
+def cpu_baseline(target_s: float = 10.0):
+    rows = calibrate_rows(target_s)
+    t, threads = cpu_oracle_gemm(rows)
+    ops = 2.0 * rows * N * K
+    return {"value": ops / t / 1e12, "unit": "TOPS", "cores": threads, "kind": "oracle",
+            "sample": f"{rows} of {M} rows of the {M}^3 product (C[rows,:] = A[rows,:] B), "
+                      f"{t:.1f} s on {threads} threads, plain C int64 loops"}
+
+
+# ------------------------------------------------------------------ timing
+def event_pair(torch):
+    return torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+
+def op_times(torch, make_plan, call, ops, reps, dev):
+    """Setup / cached steady-state / execute-only times of one operator
+    (paper: Methodology, Table 2 QPU-C and QPU-E columns)."""
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    plan = make_plan()
+    call(plan)
+    torch.cuda.synchronize(dev)
+    setup_ms = (time.perf_counter() - t0) * 1e3
+    for _ in range(3):
+        call(plan)
+    torch.cuda.synchronize(dev)
+    cached = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        call(plan)
+        torch.cuda.synchronize(dev)
+        cached.append((time.perf_counter() - t0) * 1e3)
+    execs = []
+    for _ in range(reps):
+        s, e = event_pair(torch)
+        s.record()
+        call(plan)
+        e.record()
+        e.synchronize()
+        execs.append(s.elapsed_time(e))
+    st = plan.status()
+    plan.close()
+    c = statistics.median(cached)
+    x = statistics.median(execs)
+    return {"setup_ms": round(setup_ms, 3), "cached_ms": round(c, 4), "execute_ms": round(x, 4),
+            "cached_gops": round(ops / (c * 1e-3) / 1e9, 1),
+            "execute_gops": round(ops / (x * 1e-3) / 1e9, 1), "status": st}
+
+
+def operators(torch, qx, inputs, dev):
+    out = {}
+    x, w = inputs.conv_case(8, 64, 56, 56, 128, 3, 3, -255, 255, seed=0)
+    x, w = x.to(dev), w.to(dev)
+    y = torch.empty((8, 128, 56, 56), dtype=torch.int32, device=dev)
+    conv_ops = 2.0 * 8 * 128 * 56 * 56 * 64 * 9
+    out["conv_int16"] = op_times(
+        torch, lambda: qx.Plan(qx.conv_desc(8, 64, 56, 56, 128, 3, 3, 1, 1, (-255, 255), (-255, 255))),
+        lambda p: p.conv2d(x, w, y), conv_ops, 50, dev)
+    out["conv_int16"]["workload"] = "x 8x64x56x56, w 128x64x3x3, stride 1 pad 1, int16 in [-255,255]"
+    xi, wi = x.to(torch.int32), w.to(torch.int32)
+    out["conv_int32"] = op_times(
+        torch, lambda: qx.Plan(qx.conv_desc(8, 64, 56, 56, 128, 3, 3, 1, 1, (-255, 255), (-255, 255),
+                                            dtype=qx.I32)),
+        lambda p: p.conv2d(xi, wi, y), conv_ops, 50, dev)
+    Q, Kt, V = (t.to(dev) for t in inputs.attn_case(1024, 64, -7, 7, seed=0))
+    O = torch.empty((1024, 64), dtype=torch.int32, device=dev)
+    attn_ops = 4.0 * 1024 * 1024 * 64
+    out["attn_int16"] = op_times(
+        torch, lambda: qx.Plan(qx.attn_desc(1024, 64, (-7, 7), (-7, 7), (-7, 7))),
+        lambda p: p.attn(Q, Kt, V, O), attn_ops, 50, dev)
+    out["attn_int16"]["workload"] = "Q,K,V 1024x64 int16 in [-7,7], O=(QK^T)V, no softmax"
+    Qi, Ki, Vi = (t.to(torch.int32) for t in (Q, Kt, V))
+    out["attn_int32"] = op_times(
+        torch, lambda: qx.Plan(qx.attn_desc(1024, 64, (-7, 7), (-7, 7), (-7, 7), dtype=qx.I32)),
+        lambda p: p.attn(Qi, Ki, Vi, O), attn_ops, 50, dev)
+    return out
+
+
+# -------------------------------------------------------------------- main
+def run_reference(args):
+    rank = _env_int("RANK", 0)
+    if rank != 0:
+        return 0
+    steps, warmup = args.steps, args.warmup
+    # size each step so warm-up + timed steps take about two minutes in all
+    per_step_s = max(0.5, 120.0 / max(1, steps + warmup))
+    rows = calibrate_rows(per_step_s)
+    for _ in range(warmup):
+        cpu_oracle_gemm(rows)
+    times = []
+    threads = 1
+    for _ in range(steps):
+        t, threads = cpu_oracle_gemm(rows)
+        times.append(t)
+    t_step = sum(times) / len(times)
+    value = 2.0 * rows * N * K / t_step / 1e12
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS",
+            "n_gpus": args.gpus, "steps": steps, "warmup": warmup,
+            "ms_per_step": t_step * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": {"workload": workload_name(), "sample_rows": rows},
+            "cpu_baseline": {"value": value, "unit": "TOPS", "cores": threads, "kind": "oracle",
+                             "sample": f"{rows} of {M} rows of the {M}^3 product per step"},
+            "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_qx(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2606_09905_gb300 import _build
+    _build.build()
+    from paper_2606_09905_gb300 import inputs, qx
+
+    world = _env_int("WORLD_SIZE", 1)
+    rank = _env_int("RANK", 0)
+    local = _env_int("LOCAL_RANK", 0)
+    if world != args.gpus and world > 1:
+        raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE {world}")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    A, B = inputs.gemm_case(M, N, K, LO, HI, seed=rank)
+    dA, dB = A.to(dev), B.to(dev)
+    C = torch.empty((M, N), dtype=torch.int32, device=dev)
+    desc = qx.gemm_desc(M, N, K, (LO, HI), (LO, HI))
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    plan = qx.Plan(desc, device=local)
+    plan.gemm_i16_i32(dA, dB, C)
+    torch.cuda.synchronize(dev)
+    setup_ms = (time.perf_counter() - t0) * 1e3
+    scheme = plan.info()[0]
+    m_limb = scheme["mma_per_kstep"]
+
+    for _ in range(args.warmup):
+        plan.pack(dA, dB)
+        plan.run_packed(C)
+    torch.cuda.synchronize(dev)
+
+    # ---------------------------------------------------------- timed region
+    stream = torch.cuda.current_stream(dev)
+    marks = [event_pair(torch) for _ in range(args.steps)]
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    t_start, t_stop = event_pair(torch)
+    sampler = ClockSampler(gpu_smi_id(torch, local))
+    sampler.start()
+    barrier()
+    torch.cuda.synchronize(dev)
+    t_start.record(stream)
+    for i in range(args.steps):
+        starts[i].record(stream)
+        plan.pack(dA, dB)
+        marks[i][0].record(stream)
+        plan.run_packed(C)
+        marks[i][1].record(stream)
+    t_stop.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier()
+    clocks = sampler.stop()
+    ms_total = t_start.elapsed_time(t_stop)
+    if world > 1:
+        tt = torch.tensor([ms_total], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms_total = float(tt.item())
+    ms_step = ms_total / args.steps
+    kernel_ms = statistics.mean(m[0].elapsed_time(m[1]) for m in marks)
+    pack_ms = statistics.mean(s.elapsed_time(m[0]) for s, m in zip(starts, marks))
+    st = plan.status()
+    if st != qx.OK:
+        raise SystemExit(f"device status {st} after the timed region")
+
+    ops = 2.0 * M * N * K
+    value = world * ops / (ms_step * 1e-3) / 1e12
+
+    # -------------------------------------------- end to end, host buffers
+    hA = A.pin_memory()
+    hB = B.pin_memory()
+    hC = torch.empty((M, N), dtype=torch.int32).pin_memory()
+    e2e_steps = max(3, min(args.steps, 10))
+    for _ in range(2):
+        dA.copy_(hA, non_blocking=True)
+        dB.copy_(hB, non_blocking=True)
+        plan.gemm_i16_i32(dA, dB, C)
+        hC.copy_(C, non_blocking=True)
+    torch.cuda.synchronize(dev)
+    barrier()
+    e0, e1 = event_pair(torch)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        dA.copy_(hA, non_blocking=True)
+        dB.copy_(hB, non_blocking=True)
+        plan.gemm_i16_i32(dA, dB, C)
+        hC.copy_(C, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    if world > 1:
+        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    e2e = {"value": world * ops / (e2e_ms * 1e-3) / 1e12, "unit": "TOPS",
+           "h2d_bytes_per_step": hA.numel() * 2 + hB.numel() * 2,
+           "d2h_bytes_per_step": hC.numel() * 4, "ms_per_step": e2e_ms}
+
+    # cached steady state (host wall per call, with sync), as the paper's QPU-C
+    cached = []
+    for _ in range(5):
+        t0 = time.perf_counter()
+        plan.gemm_i16_i32(dA, dB, C)
+        torch.cuda.synchronize(dev)
+        cached.append((time.perf_counter() - t0) * 1e3)
+
+    peaks = load_peaks()
+    flops_launch = m_limb * 2.0 * M * N * K          # FP16 tensor work of the exact scheme
+    achieved = flops_launch / (kernel_ms * 1e-3) / 1e12
+    # a timed loop of a second or more runs under the power cap: compare it
+    # with the sustained peak; shorter bursts with the burst peak
+    long_run = ms_total >= 1000.0
+    peak = peaks["bf16_tflops_sustained"] if long_run else peaks["bf16_tflops"]
+    peak_kind = "sustained" if long_run else "burst"
+    pack_bytes = (M * K + K * N) * 2 + (scheme["limbs_a"] * M * K + scheme["limbs_b"] * N * K) * 2
+    roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
+                "frac": round(achieved / peak, 4), "traffic": None,
+                "kernel": "qx::limb_gemm_kernel<2,1>", "kernel_ms": round(kernel_ms, 4),
+                "peak_source": f"{peaks['source']} dense bf16 {peak_kind} (FP16 runs at the BF16 rate); "
+                               f"timed loop {ms_total / 1e3:.2f} s",
+                "frac_of_burst": round(achieved / peaks["bf16_tflops"], 4),
+                "flops_per_launch": flops_launch,
+                "int_tops_roofline": round(peak / m_limb, 1),
+                "int_tops_kernel": round(ops / (kernel_ms * 1e-3) / 1e12, 1),
+                "pack_kernel": {"ms": round(pack_ms, 4),
+                                "gbs": round(pack_bytes / (pack_ms * 1e-3) / 1e9, 1),
+                                "hbm_peak_gbs": peaks["hbm_gbs"]}}
+
+    extras = {}
+    if not args.no_operators:
+        extras = operators(torch, qx, inputs, dev)
+    extras[f"gemm{M}"] = {"setup_ms": round(setup_ms, 2), "cached_ms": round(statistics.median(cached), 4),
+                          "execute_ms": round(ms_step, 4),
+                          "cached_tops": round(ops / (statistics.median(cached) * 1e-3) / 1e12, 1),
+                          "execute_tops": round(ops / (ms_step * 1e-3) / 1e12, 1)}
+    plan.close()
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cpu = cpu_baseline(args.cpu_seconds)
+
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    if rank != 0:
+        return 0
+    line = {"metric": METRIC, "value": round(value, 2), "unit": "TOPS", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "i16->i32", "data": "synthetic",
+            "config": {"workload": workload_name(), "M": M, "N": N, "K": K,
+                       "l2": "inputs larger than L2 (A, B 128 MiB each; limb planes 384 MiB; C 256 MiB)",
+                       "scheme": scheme, "parallelism": f"replicas x{world}"},
+            "e2e": e2e, "roofline": roofline, "cpu_baseline": cpu,
+            "gpu_launches": 2 * args.steps, "clocks": clocks, "operators": extras}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["qx", "reference"], default="qx")
+    ap.add_argument("--no-operators", action="store_true", help="skip the conv/attention timings")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--size", type=int, default=8192,
+                    help="M = N = K of the GEMM step (8192 is the benchmark workload; smaller "
+                         "sizes exist for profiling captures)")
+    args = ap.parse_args()
+    global M, N, K
+    M = N = K = args.size
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be at least 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_qx(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -153,6 +153,18 @@ qx_status qx_conv2d_gemm(qx_plan plan, const void *x, const void *w, void *y,
 qx_status qx_attn_core(qx_plan plan, const void *Q, const void *K,
                        const void *V, void *O, qx_stream stream);
 
+/* The two halves of every execution call above, for callers that time or
+ * overlap them separately (paper: Methodology and Table 2 separate cached
+ * steady-state from execute-only time).  qx_pack rewrites the operands into
+ * the plan's FP16 limb workspace: GEMM a = A, b = B; Conv2D a = x, b = w;
+ * attention a = Q, b = K, c = V (c is ignored otherwise).  qx_run_packed
+ * runs the tensor-core kernel on that workspace and writes the output
+ * (C, y or O).  qx_pack followed by qx_run_packed on one stream is exactly
+ * the combined call.  Same pointer, alignment and ownership rules. */
+qx_status qx_pack(qx_plan plan, const void *a, const void *b, const void *c,
+                  qx_stream stream);
+qx_status qx_run_packed(qx_plan plan, void *out, qx_stream stream);
+
 /* Synchronises the plan's device, then returns and clears the sticky device
  * error word (QX_ERR_TIMEOUT or QX_ERR_CONTRACT), or QX_OK. */
 qx_status qx_plan_status(qx_plan plan);

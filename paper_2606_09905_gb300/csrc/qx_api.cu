@@ -566,87 +566,139 @@ qx_status qx_plan_status(qx_plan p) {
 
 static bool aligned16(const void *ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
 
-static qx_status run_gemm(qx_plan p, const void *A, const void *B, int32_t *C, cudaStream_t stream,
-                          qx_dtype want) {
+static const char *op_name(qx_op op) {
+    return op == QX_OP_GEMM ? "GEMM" : op == QX_OP_CONV2D ? "conv" : "attention";
+}
+
+// Operand packing: operands -> FP16 limb planes in the workspace.
+static qx_status pack(qx_plan p, const void *a, const void *b, const void *c, cudaStream_t st) {
+    const qx_plan_desc &d = p->desc;
+    const int check = (d.flags & QX_FLAG_CHECK_RANGES) ? 1 : 0;
+    const bool i32 = d.in_dtype == QX_I32;
+    switch (d.op) {
+        case QX_OP_GEMM: {
+            if (d.M == 0 || d.N == 0 || d.K == 0) return QX_OK;
+            if (!a || !b) return fail(QX_ERR_INVALID_ARG, "null operand");
+            if (!aligned16(a) || !aligned16(b))
+                return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+            const Scheme &s = p->scheme[0];
+            QX_CUDA(launch_pack_gemm(i32, a, b, d.lda, d.ldb, int(d.M), int(d.N), int(d.K), p->Kp,
+                                     p->planes_n, p->planes_m, s.n.limbs, s.n.shift, s.m.limbs,
+                                     s.m.shift, check, d.range_a, d.range_b, p->err, p->num_sms, st),
+                    "operand packing launch");
+            return QX_OK;
+        }
+        case QX_OP_CONV2D: {
+            if (!a || !b) return fail(QX_ERR_INVALID_ARG, "null operand");
+            if (!aligned16(a) || !aligned16(b))
+                return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+            const Scheme &s = p->scheme[0];
+            QX_CUDA(launch_pack_conv(i32, a, b, int(d.n), int(d.c), int(d.h), int(d.w),
+                                     int(d.k_out), int(d.r), int(d.s), p->Cp, p->planes_m,
+                                     p->planes_n, s.m.limbs, s.m.shift, s.n.limbs, s.n.shift, check,
+                                     d.range_a, d.range_b, p->err, p->num_sms, st),
+                    "operand packing launch");
+            return QX_OK;
+        }
+        case QX_OP_ATTN: {
+            if (!a || !b || !c) return fail(QX_ERR_INVALID_ARG, "null operand");
+            if (!aligned16(a) || !aligned16(b) || !aligned16(c))
+                return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+            QX_CUDA(launch_pack_attn(i32, a, b, c, int(d.L), int(d.d), p->dp, p->Lp, p->aq, p->ak,
+                                     p->avt, check, d.range_a, d.range_b, d.range_c, p->err,
+                                     p->num_sms, st),
+                    "operand packing launch");
+            return QX_OK;
+        }
+    }
+    return fail(QX_ERR_INVALID_ARG, "unknown op");
+}
+
+// The tensor-core kernel on the packed workspace.
+static qx_status run_packed(qx_plan p, void *out, cudaStream_t st) {
+    const qx_plan_desc &d = p->desc;
+    if (!out) return fail(QX_ERR_INVALID_ARG, "null output");
+    if (!aligned16(out)) return fail(QX_ERR_UNSUPPORTED, "output must be 16-byte aligned");
+    switch (d.op) {
+        case QX_OP_GEMM: {
+            if (d.M == 0 || d.N == 0) return QX_OK;
+            if (d.K == 0) {
+                QX_CUDA(cudaMemset2DAsync(out, size_t(d.ldc) * 4, 0, size_t(d.N) * 4, size_t(d.M), st),
+                        "zero output");
+                return QX_OK;
+            }
+            MmaArgs a = p->mma;
+            a.out = static_cast<int32_t *>(out);
+            QX_CUDA(limb_gemm_launch(p->scheme[0].n.limbs, p->scheme[0].m.limbs, a, p->grid, st),
+                    "limb GEMM launch");
+            return QX_OK;
+        }
+        case QX_OP_CONV2D: {
+            MmaArgs a = p->mma;
+            a.out = static_cast<int32_t *>(out);
+            QX_CUDA(limb_gemm_launch(p->scheme[0].n.limbs, p->scheme[0].m.limbs, a, p->grid, st),
+                    "conv launch");
+            return QX_OK;
+        }
+        case QX_OP_ATTN: {
+            QX_CUDA(cudaMemsetAsync(out, 0, size_t(d.L) * d.d * 4, st), "zero output");
+            AttnArgs a = p->attn;
+            a.out = static_cast<int32_t *>(out);
+            QX_CUDA(attn_launch(a, st), "attention launch");
+            return QX_OK;
+        }
+    }
+    return fail(QX_ERR_INVALID_ARG, "unknown op");
+}
+
+static qx_status execute(qx_plan p, qx_op op, qx_dtype want, const void *a, const void *b,
+                         const void *c, void *out, qx_stream stream) {
     if (!p) return fail(QX_ERR_INVALID_ARG, "null plan");
     const qx_plan_desc &d = p->desc;
-    if (d.op != QX_OP_GEMM || d.in_dtype != want)
-        return fail(QX_ERR_INVALID_ARG, "plan is not a %s GEMM plan", want == QX_I16 ? "I16" : "I32");
-    if (d.M == 0 || d.N == 0) return QX_OK;
-    if (!C || (d.K > 0 && (!A || !B))) return fail(QX_ERR_INVALID_ARG, "null operand");
-    if (!aligned16(C) || (d.K > 0 && (!aligned16(A) || !aligned16(B))))
-        return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+    if (d.op != op) return fail(QX_ERR_INVALID_ARG, "plan is not a %s plan", op_name(op));
+    if (op == QX_OP_GEMM && d.in_dtype != want)
+        return fail(QX_ERR_INVALID_ARG, "plan is not an %s GEMM plan", want == QX_I16 ? "I16" : "I32");
     DeviceScope scope;
     QX_CUDA(scope.enter(p->device), "cudaSetDevice");
-    if (d.K == 0) {
-        QX_CUDA(cudaMemset2DAsync(C, size_t(d.ldc) * 4, 0, size_t(d.N) * 4, size_t(d.M), stream),
-                "zero output");
-        return QX_OK;
-    }
-    const Scheme &s = p->scheme[0];
-    QX_CUDA(launch_pack_gemm(want == QX_I32, A, B, d.lda, d.ldb, int(d.M), int(d.N), int(d.K),
-                             p->Kp, p->planes_n, p->planes_m, s.n.limbs, s.n.shift, s.m.limbs,
-                             s.m.shift, (d.flags & QX_FLAG_CHECK_RANGES) ? 1 : 0, d.range_a,
-                             d.range_b, p->err, p->num_sms, stream),
-            "operand packing launch");
-    MmaArgs a = p->mma;
-    a.out = C;
-    QX_CUDA(limb_gemm_launch(s.n.limbs, s.m.limbs, a, p->grid, stream), "limb GEMM launch");
-    return QX_OK;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (op == QX_OP_GEMM && (d.M == 0 || d.N == 0)) return QX_OK;
+    if (!out) return fail(QX_ERR_INVALID_ARG, "null output");
+    if (!aligned16(out)) return fail(QX_ERR_UNSUPPORTED, "output must be 16-byte aligned");
+    qx_status s = pack(p, a, b, c, st);
+    if (s != QX_OK) return s;
+    return run_packed(p, out, st);
 }
 
 qx_status qx_gemm_i16_i32(qx_plan p, const int16_t *A, const int16_t *B, int32_t *C,
                           qx_stream stream) {
-    return run_gemm(p, A, B, C, reinterpret_cast<cudaStream_t>(stream), QX_I16);
+    return execute(p, QX_OP_GEMM, QX_I16, A, B, nullptr, C, stream);
 }
 
 qx_status qx_gemm_i32(qx_plan p, const int32_t *A, const int32_t *B, int32_t *C, qx_stream stream) {
-    return run_gemm(p, A, B, C, reinterpret_cast<cudaStream_t>(stream), QX_I32);
+    return execute(p, QX_OP_GEMM, QX_I32, A, B, nullptr, C, stream);
 }
 
 qx_status qx_conv2d_gemm(qx_plan p, const void *x, const void *w, void *y, qx_stream stream) {
-    if (!p) return fail(QX_ERR_INVALID_ARG, "null plan");
-    const qx_plan_desc &d = p->desc;
-    if (d.op != QX_OP_CONV2D) return fail(QX_ERR_INVALID_ARG, "plan is not a conv plan");
-    if (!x || !w || !y) return fail(QX_ERR_INVALID_ARG, "null operand");
-    if (!aligned16(x) || !aligned16(w) || !aligned16(y))
-        return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
-    DeviceScope scope;
-    QX_CUDA(scope.enter(p->device), "cudaSetDevice");
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    const Scheme &s = p->scheme[0];
-    QX_CUDA(launch_pack_conv(d.in_dtype == QX_I32, x, w, int(d.n), int(d.c), int(d.h), int(d.w),
-                             int(d.k_out), int(d.r), int(d.s), p->Cp, p->planes_m, p->planes_n,
-                             s.m.limbs, s.m.shift, s.n.limbs, s.n.shift,
-                             (d.flags & QX_FLAG_CHECK_RANGES) ? 1 : 0, d.range_a, d.range_b,
-                             p->err, p->num_sms, st),
-            "operand packing launch");
-    MmaArgs a = p->mma;
-    a.out = static_cast<int32_t *>(y);
-    QX_CUDA(limb_gemm_launch(s.n.limbs, s.m.limbs, a, p->grid, st), "conv launch");
-    return QX_OK;
+    return execute(p, QX_OP_CONV2D, QX_I16, x, w, nullptr, y, stream);
 }
 
 qx_status qx_attn_core(qx_plan p, const void *Q, const void *K, const void *V, void *O,
                        qx_stream stream) {
+    return execute(p, QX_OP_ATTN, QX_I16, Q, K, V, O, stream);
+}
+
+qx_status qx_pack(qx_plan p, const void *a, const void *b, const void *c, qx_stream stream) {
     if (!p) return fail(QX_ERR_INVALID_ARG, "null plan");
-    const qx_plan_desc &d = p->desc;
-    if (d.op != QX_OP_ATTN) return fail(QX_ERR_INVALID_ARG, "plan is not an attention plan");
-    if (!Q || !K || !V || !O) return fail(QX_ERR_INVALID_ARG, "null operand");
-    if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
-        return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
     DeviceScope scope;
     QX_CUDA(scope.enter(p->device), "cudaSetDevice");
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    QX_CUDA(cudaMemsetAsync(O, 0, size_t(d.L) * d.d * 4, st), "zero output");
-    QX_CUDA(launch_pack_attn(d.in_dtype == QX_I32, Q, K, V, int(d.L), int(d.d), p->dp, p->Lp,
-                             p->aq, p->ak, p->avt, (d.flags & QX_FLAG_CHECK_RANGES) ? 1 : 0,
-                             d.range_a, d.range_b, d.range_c, p->err, p->num_sms, st),
-            "operand packing launch");
-    AttnArgs a = p->attn;
-    a.out = static_cast<int32_t *>(O);
-    QX_CUDA(attn_launch(a, st), "attention launch");
-    return QX_OK;
+    return pack(p, a, b, c, reinterpret_cast<cudaStream_t>(stream));
+}
+
+qx_status qx_run_packed(qx_plan p, void *out, qx_stream stream) {
+    if (!p) return fail(QX_ERR_INVALID_ARG, "null plan");
+    DeviceScope scope;
+    QX_CUDA(scope.enter(p->device), "cudaSetDevice");
+    return run_packed(p, out, reinterpret_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"

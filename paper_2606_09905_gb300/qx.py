@@ -27,7 +27,8 @@ FLAG_CHECK_RANGES = 1
 # Every function the header declares; the CPU tests check the exports.
 EXPORTS = ("qx_plan_create", "qx_plan_destroy", "qx_plan_query", "qx_plan_info",
            "qx_gemm_i16_i32", "qx_gemm_i32", "qx_conv2d_gemm", "qx_attn_core",
-           "qx_plan_status", "qx_status_string", "qx_last_error", "qx_version")
+           "qx_pack", "qx_run_packed", "qx_plan_status", "qx_status_string",
+           "qx_last_error", "qx_version")
 
 
 class QxError(RuntimeError):
@@ -87,6 +88,8 @@ def load() -> ctypes.CDLL:
             "qx_gemm_i32": ([P, V, V, V, V], ctypes.c_int),
             "qx_conv2d_gemm": ([P, V, V, V, V], ctypes.c_int),
             "qx_attn_core": ([P, V, V, V, V, V], ctypes.c_int),
+            "qx_pack": ([P, V, V, V, V], ctypes.c_int),
+            "qx_run_packed": ([P, V, V], ctypes.c_int),
             "qx_plan_status": ([P], ctypes.c_int),
             "qx_status_string": ([ctypes.c_int], ctypes.c_char_p),
             "qx_last_error": ([], ctypes.c_char_p),
@@ -201,6 +204,16 @@ class Plan:
         n = ctypes.c_int(0)
         _check(load().qx_plan_info(self.handle, out, ctypes.byref(n)), "qx_plan_info")
         return [out[i].as_dict() for i in range(n.value)]
+
+    # -- the two halves of an execution (pack, then the tensor-core kernel) --
+    def pack(self, a, b, c=None, stream=None):
+        lib = load()
+        ptr = lambda t: None if t is None else t.data_ptr()
+        _check(lib.qx_pack(self.handle, ptr(a), ptr(b), ptr(c), _stream(stream)), "qx_pack")
+
+    def run_packed(self, out, stream=None):
+        _check(load().qx_run_packed(self.handle, out.data_ptr(), _stream(stream)), "qx_run_packed")
+        return out
 
     def status(self) -> int:
         """Synchronise and return (and clear) the device error word as a status."""
