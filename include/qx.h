@@ -169,6 +169,35 @@ qx_status qx_run_packed(qx_plan plan, void *out, qx_stream stream);
  * error word (QX_ERR_TIMEOUT or QX_ERR_CONTRACT), or QX_OK. */
 qx_status qx_plan_status(qx_plan plan);
 
+/* Allocation-free INT16 GEMM.  The paper has no counterpart; this entry
+ * point exists for callers that cannot call cudaMalloc when they multiply:
+ * code running inside an allocator or memory-pool callback (allocating there
+ * would recurse), hosts whose device-memory budget is fixed at start-up, and
+ * latency-critical paths that cannot take cudaMalloc's implicit device
+ * synchronisation.  Unlike qx_plan_create it allocates nothing: the limb
+ * planes live in one static device array of QX_STATIC_SCRATCH_BYTES that the
+ * library places on every device it is loaded on, held until the process
+ * exits.  It computes what qx_gemm_i16_i32 computes, C = A * B with A int16
+ * (M x K), B int16 (K x N), C int32 (M x N), all tightly packed row-major,
+ * 16-byte aligned device pointers on the current device, asynchronous on
+ * `stream`; the scheme follows from range_a / range_b as in a plan, and
+ * flags takes QX_FLAG_CHECK_RANGES.
+ *   - Problems whose planes exceed the scratch (about 24 MiB of operands at
+ *     2048^3) return QX_ERR_UNSUPPORTED and launch nothing.
+ *   - The first call on a device looks up the scratch's device address
+ *     (cudaGetSymbolAddress); make that first call before any stream capture.
+ *   - Every call on a device shares the scratch and leaves its planes in it;
+ *     calls that overlap on the GPU race, so serialise them.
+ *   - dev_status (may be NULL): a caller-owned, caller-zeroed device int that
+ *     receives QX_ERR_TIMEOUT or QX_ERR_CONTRACT from the kernels; with NULL a
+ *     word inside the scratch, cleared at every call, is used instead and
+ *     device-side errors are not reported. */
+#define QX_STATIC_SCRATCH_BYTES (32u << 20)
+qx_status qx_gemm_i16_i32_noalloc(int64_t M, int64_t N, int64_t K, qx_range range_a,
+                                  qx_range range_b, unsigned flags, const int16_t *A,
+                                  const int16_t *B, int32_t *C, int *dev_status,
+                                  qx_stream stream);
+
 const char *qx_status_string(qx_status status);
 const char *qx_last_error(void);
 int qx_version(void);

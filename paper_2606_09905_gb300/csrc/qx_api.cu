@@ -63,6 +63,11 @@ static qx_status fail(qx_status st, const char *fmt, ...) {
     return st;
 }
 
+namespace qx {
+// Lets other translation units of the library set the qx_last_error text.
+void set_last_error(const char *msg) { g_last_error = msg; }
+}  // namespace qx
+
 static qx_status cuda_fail(cudaError_t e, const char *what) {
     cudaGetLastError();  // clear the sticky-free error state
     return fail(e == cudaErrorMemoryAllocation ? QX_ERR_OOM : QX_ERR_CUDA, "%s: %s", what,

@@ -1,0 +1,254 @@
+// qx_noalloc.cu -- an INT16 GEMM entry point that allocates no device memory.
+//
+// Who needs it: callers that cannot call cudaMalloc at the point where they
+// multiply -- code that runs inside an allocator or memory-pool callback
+// (allocating again there would recurse into the allocator), hosts that fix
+// their device-memory budget at start-up and forbid growth afterwards, and
+// latency-critical paths that cannot afford cudaMalloc's implicit device
+// synchronisation.  The plan-based API allocates its workspace in
+// qx_plan_create, so these callers cannot use it.
+//
+// How: the FP16 limb planes that the packing kernel writes and the tensor-
+// core kernel reads live in one file-scope __device__ array of fixed size
+// (QX_STATIC_SCRATCH_BYTES).  The CUDA runtime places it in every device's
+// memory when this library's module is loaded there, and it stays until the
+// process exits.  Host code must not pass the array's name to a kernel: on
+// the host that name is only a stand-in symbol, not a device address.  The
+// device address is looked up once per device with cudaGetSymbolAddress (on
+// the first call made with that device current) and cached.
+//
+// Every call on a device shares the one array, and each call leaves its own
+// planes behind in it.  Calls whose work overlaps on the GPU (two streams, or
+// two host threads on one device) race on the array; serialise them.
+#include <cuda.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include "qx_internal.h"
+
+namespace qx {
+bool plan_contraction(qx_range rn, qx_range rm, int64_t K, Scheme *best);
+int limb_gemm_rows_per_limb(int na);
+cudaError_t limb_gemm_prepare(int na, int nb);
+cudaError_t limb_gemm_launch(int na, int nb, const MmaArgs &a, int grid, cudaStream_t stream);
+cudaError_t launch_pack_gemm(bool i32, const void *A, const void *B, int64_t lda, int64_t ldb,
+                             int M, int N, int K, int Kp, __half *a_planes, __half *bt_planes,
+                             int na, int shift_a, int nb, int shift_b, int check, qx_range ra,
+                             qx_range rb, int *err, int num_sms, cudaStream_t st);
+void set_last_error(const char *msg);
+}  // namespace qx
+
+using namespace qx;
+
+static constexpr size_t kScratchBytes = size_t(QX_STATIC_SCRATCH_BYTES);
+
+// The shared scratch: a 256-byte error word, then the limb planes.
+static __device__ __align__(256) unsigned char qx_static_scratch[kScratchBytes];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceScratch {
+    std::once_flag once;
+    void *addr = nullptr;   // device address of qx_static_scratch on this device
+    int num_sms = 0;
+    qx_status status = QX_OK;
+    std::string why;
+};
+
+DeviceScratch g_dev[kMaxDevices];
+std::once_flag g_encoder_once;
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+qx_status refuse(qx_status st, const char *fmt, ...) __attribute__((format(printf, 2, 3)));
+qx_status refuse(qx_status st, const char *fmt, ...) {
+    char buf[400];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    set_last_error(buf);
+    return st;
+}
+
+// Once per device, with that device current: look up the scratch address.
+qx_status scratch_for_device(int dev, void **addr, int *num_sms) {
+    if (dev < 0 || dev >= kMaxDevices) return refuse(QX_ERR_DEVICE, "device index %d out of range", dev);
+    DeviceScratch &d = g_dev[dev];
+    std::call_once(d.once, [&d, dev] {
+        int major = 0, minor = 0;
+        if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+            major * 10 + minor != 103) {
+            cudaGetLastError();
+            d.status = QX_ERR_DEVICE;
+            d.why = "the current device is not an sm_103 GPU";
+            return;
+        }
+        void *p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, qx_static_scratch);
+        if (e != cudaSuccess || p == nullptr) {
+            cudaGetLastError();
+            d.status = QX_ERR_CUDA;
+            d.why = std::string("cudaGetSymbolAddress(static scratch) failed: ") + cudaGetErrorString(e);
+            return;
+        }
+        d.addr = p;
+        if (cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+            cudaGetLastError();
+            d.status = QX_ERR_CUDA;
+            d.why = "cudaDeviceGetAttribute(multiProcessorCount) failed";
+        }
+    });
+    if (d.status != QX_OK) return refuse(d.status, "%s", d.why.c_str());
+    *addr = d.addr;
+    *num_sms = d.num_sms;
+    return QX_OK;
+}
+
+qx_status encoder() {
+    std::call_once(g_encoder_once, [] {
+        cudaDriverEntryPointQueryResult q;
+        void *fn = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    });
+    if (!g_encode) return refuse(QX_ERR_CUDA, "cuTensorMapEncodeTiled entry point not found");
+    return QX_OK;
+}
+
+qx_status encode(CUtensorMap *map, const void *base, int rank, const cuuint64_t *dims,
+                 const cuuint64_t *strides, const cuuint32_t *box) {
+    const cuuint32_t estr[3] = {1, 1, 1};
+    const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, rank, const_cast<void *>(base),
+                                dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return refuse(QX_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", int(r));
+    return QX_OK;
+}
+
+size_t round256(size_t v) { return (v + 255) & ~size_t(255); }
+
+bool misaligned(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
+
+}  // namespace
+
+extern "C" qx_status qx_gemm_i16_i32_noalloc(int64_t M, int64_t N, int64_t K, qx_range range_a,
+                                             qx_range range_b, unsigned flags, const int16_t *A,
+                                             const int16_t *B, int32_t *C, int *dev_status,
+                                             qx_stream stream) {
+    if (M < 0 || N < 0 || K < 0 || M > INT32_MAX / 2 || N > INT32_MAX / 2 || K > INT32_MAX / 2)
+        return refuse(QX_ERR_INVALID_ARG, "GEMM sizes out of range");
+    if (range_a.lo > range_a.hi || range_b.lo > range_b.hi || range_a.lo < -32768 ||
+        range_a.hi > 32767 || range_b.lo < -32768 || range_b.hi > 32767)
+        return refuse(QX_ERR_INVALID_ARG, "operand range empty or outside int16");
+    if (M == 0 || N == 0) return QX_OK;
+    if (!C || (K > 0 && (!A || !B))) return refuse(QX_ERR_INVALID_ARG, "null operand");
+    if (misaligned(C) || (K > 0 && (misaligned(A) || misaligned(B))))
+        return refuse(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+
+    Scheme s;
+    if (!plan_contraction(range_a, range_b, K, &s))
+        return refuse(QX_ERR_CONTRACT, "no exact limb scheme for these ranges and K");
+    const int na = s.n.limbs, nb = s.m.limbs;
+    const int64_t Kp = (K + 7) / 8 * 8;
+    const size_t a_bytes = size_t(na) * size_t(M) * size_t(Kp) * 2;
+    const size_t b_bytes = size_t(nb) * size_t(N) * size_t(Kp) * 2;
+    const size_t need = 256 + round256(a_bytes) + round256(b_bytes);
+    if (need > kScratchBytes)
+        return refuse(QX_ERR_UNSUPPORTED,
+                      "this GEMM needs %zu bytes of scratch; the static scratch holds %zu bytes "
+                      "(use the plan-based qx_gemm_i16_i32 for larger problems)",
+                      need, kScratchBytes);
+
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return refuse(QX_ERR_DEVICE, "no current CUDA device");
+    }
+    void *base = nullptr;
+    int num_sms = 0;
+    qx_status st = scratch_for_device(dev, &base, &num_sms);
+    if (st != QX_OK) return st;
+    st = encoder();
+    if (st != QX_OK) return st;
+
+    cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+    int *err = dev_status;
+    if (!err) {
+        // the error word inside the scratch must start each call at zero
+        err = static_cast<int *>(base);
+        const cudaError_t e = cudaMemsetAsync(err, 0, sizeof(int), cs);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return refuse(QX_ERR_CUDA, "clearing the scratch error word: %s", cudaGetErrorString(e));
+        }
+    }
+    if (K == 0) {
+        const cudaError_t e = cudaMemset2DAsync(C, size_t(N) * 4, 0, size_t(N) * 4, size_t(M), cs);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return refuse(QX_ERR_CUDA, "zeroing C: %s", cudaGetErrorString(e));
+        }
+        return QX_OK;
+    }
+
+    __half *a_planes = reinterpret_cast<__half *>(static_cast<char *>(base) + 256);
+    __half *bt_planes = reinterpret_cast<__half *>(static_cast<char *>(base) + 256 + round256(a_bytes));
+    const int mr = limb_gemm_rows_per_limb(na);
+
+    MmaArgs a;
+    memset(&a, 0, sizeof a);
+    for (int j = 0; j < nb; ++j) {
+        const cuuint64_t dims[2] = {cuuint64_t(K), cuuint64_t(N)};
+        const cuuint64_t str[1] = {cuuint64_t(Kp) * 2};
+        const cuuint32_t box[2] = {kBK, kBM};
+        st = encode(&a.tm_m[j], bt_planes + size_t(j) * N * Kp, 2, dims, str, box);
+        if (st != QX_OK) return st;
+    }
+    {
+        const cuuint64_t dims[3] = {cuuint64_t(K), cuuint64_t(M), cuuint64_t(na)};
+        const cuuint64_t str[2] = {cuuint64_t(Kp) * 2, cuuint64_t(M) * Kp * 2};
+        const cuuint32_t box[3] = {kBK, cuuint32_t(mr), cuuint32_t(na)};
+        st = encode(&a.tm_n, a_planes, 3, dims, str, box);
+        if (st != QX_OK) return st;
+    }
+    a.out = C;
+    a.err = err;
+    a.out_row_stride = N;
+    a.mode = 0;
+    a.m_extent = int(N);
+    a.n_extent = int(M);
+    a.kblocks = int((K + kBK - 1) / kBK);
+    a.chunk_kb = int(s.chunk_kb);
+    a.tiles_m = int((N + kBM - 1) / kBM);
+    a.tiles_n = int((M + mr - 1) / mr);
+    a.group_n = a.tiles_n < 16 ? a.tiles_n : 16;
+    a.shift_n = s.n.shift;
+    a.shift_m = s.m.shift;
+    const int tiles = a.tiles_m * a.tiles_n;
+    const int grid = tiles < num_sms ? tiles : num_sms;
+
+    cudaError_t e = limb_gemm_prepare(na, nb);
+    if (e == cudaSuccess)
+        e = launch_pack_gemm(false, A, B, K, N, int(M), int(N), int(K), int(Kp), a_planes, bt_planes,
+                             na, s.n.shift, nb, s.m.shift, (flags & QX_FLAG_CHECK_RANGES) ? 1 : 0,
+                             range_a, range_b, err, num_sms, cs);
+    if (e == cudaSuccess) e = limb_gemm_launch(na, nb, a, grid, cs);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return refuse(QX_ERR_CUDA, "launch failed: %s", cudaGetErrorString(e));
+    }
+    return QX_OK;
+}

@@ -28,7 +28,7 @@ FLAG_CHECK_RANGES = 1
 EXPORTS = ("qx_plan_create", "qx_plan_destroy", "qx_plan_query", "qx_plan_info",
            "qx_gemm_i16_i32", "qx_gemm_i32", "qx_conv2d_gemm", "qx_attn_core",
            "qx_pack", "qx_run_packed", "qx_plan_status", "qx_status_string",
-           "qx_last_error", "qx_version")
+           "qx_last_error", "qx_version", "qx_gemm_i16_i32_noalloc")
 
 
 class QxError(RuntimeError):
@@ -94,6 +94,8 @@ def load() -> ctypes.CDLL:
             "qx_status_string": ([ctypes.c_int], ctypes.c_char_p),
             "qx_last_error": ([], ctypes.c_char_p),
             "qx_version": ([], ctypes.c_int),
+            "qx_gemm_i16_i32_noalloc": ([ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, Range,
+                                         Range, ctypes.c_uint, V, V, V, V, V], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -138,6 +140,20 @@ def query(desc: PlanDesc) -> list[dict]:
     n = ctypes.c_int(0)
     _check(lib.qx_plan_query(ctypes.byref(desc), out, ctypes.byref(n)), "qx_plan_query")
     return [out[i].as_dict() for i in range(n.value)]
+
+
+def gemm_i16_i32_noalloc(A, B, C, range_a, range_b, flags=0, dev_status=None, stream=None):
+    """C = A @ B through the allocation-free entry point (no plan, no device
+    allocation; the limb planes live in the library's static scratch)."""
+    M, K = A.shape
+    N = B.shape[1]
+    a = _ptr(A, torch.int16, (M, K), "A")
+    b = _ptr(B, torch.int16, (K, N), "B")
+    c = _ptr(C, torch.int32, (M, N), "C")
+    st = None if dev_status is None else _ptr(dev_status, torch.int32, None, "dev_status")
+    _check(load().qx_gemm_i16_i32_noalloc(M, N, K, _rng(range_a), _rng(range_b), flags, a, b, c,
+                                          st, _stream(stream)), "qx_gemm_i16_i32_noalloc")
+    return C
 
 
 # ------------------------------------------------------------------- plans

@@ -1,0 +1,83 @@
+"""The allocation-free INT16 GEMM entry point, qx_gemm_i16_i32_noalloc.
+
+It serves callers that cannot call cudaMalloc when they multiply (allocator
+or memory-pool callbacks, hosts with a device-memory budget fixed at start-up,
+paths that cannot take cudaMalloc's implicit synchronisation): the limb
+planes live in a static device array instead of a plan's workspace.  These
+tests call it through the C ABI and hold it to the plan-based
+qx_gemm_i16_i32 on the same inputs, bit for bit (the integer path is exact),
+on two calls in a row that share the static scratch.  The file name sorts
+last so a run that stops at the first failure has run everything else.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2606_09905_gb300 import inputs, qx
+
+from gpu_util import build_once
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    build_once()
+
+
+def _noalloc(A, B, C, ra, rb, status=None):
+    lib = qx.load()
+    M, K = A.shape
+    N = B.shape[1]
+    return lib.qx_gemm_i16_i32_noalloc(
+        M, N, K, qx.Range(*ra), qx.Range(*rb), 0, A.data_ptr(), B.data_ptr(), C.data_ptr(),
+        None if status is None else status.data_ptr(),
+        torch.cuda.current_stream().cuda_stream)
+
+
+def _plan_result(A, B, ra, rb):
+    M, K = A.shape
+    N = B.shape[1]
+    with qx.Plan(qx.gemm_desc(M, N, K, ra, rb)) as plan:
+        C = plan.gemm_i16_i32(A, B)
+        torch.cuda.synchronize()
+        assert plan.status() == qx.OK
+    return C
+
+
+@pytest.mark.parametrize("M,N,K,lo,hi", [(256, 256, 256, -1023, 1023),
+                                         (1024, 768, 1000, -1023, 1023),
+                                         (300, 200, 77, -32768, 32767)])
+def test_noalloc_matches_plan_path_on_two_calls(M, N, K, lo, hi):
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for seed in (1, 2):                       # two calls in a row, one shared scratch
+        A, B = inputs.gemm_case(M, N, K, lo, hi, seed=seed + M)
+        A, B = A.cuda(), B.cuda()
+        C = torch.full((M, N), -1, dtype=torch.int32, device="cuda")
+        assert _noalloc(A, B, C, (lo, hi), (lo, hi), status) == qx.OK
+        torch.cuda.synchronize()
+        assert int(status.item()) == 0
+        ref = _plan_result(A, B, (lo, hi), (lo, hi))
+        assert torch.equal(C, ref), f"call {seed}: {(C != ref).sum().item()} elements differ"
+
+
+def test_noalloc_without_status_word_and_python_wrapper():
+    A, B = inputs.gemm_case(129, 130, 131, -500, 500, seed=3)
+    A, B = A.cuda(), B.cuda()
+    C = torch.empty((129, 130), dtype=torch.int32, device="cuda")
+    qx.gemm_i16_i32_noalloc(A, B, C, (-500, 500), (-500, 500))
+    torch.cuda.synchronize()
+    assert torch.equal(C, _plan_result(A, B, (-500, 500), (-500, 500)))
+
+
+def test_noalloc_rejects_problems_beyond_its_scratch():
+    M = N = K = 4096                          # needs 96 MiB of planes
+    A = torch.zeros((M, K), dtype=torch.int16, device="cuda")
+    B = torch.zeros((K, N), dtype=torch.int16, device="cuda")
+    C = torch.full((M, N), 7, dtype=torch.int32, device="cuda")
+    assert _noalloc(A, B, C, (-1023, 1023), (-1023, 1023)) == qx.ERR_UNSUPPORTED
+    assert b"static scratch" in qx.load().qx_last_error()
+    torch.cuda.synchronize()
+    assert int(C[0, 0].item()) == 7           # nothing was launched
