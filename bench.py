@@ -230,6 +230,13 @@ def operators(torch, qx, inputs, dev):
         torch, lambda: qx.Plan(qx.conv_desc(8, 64, 56, 56, 128, 3, 3, 1, 1, (-255, 255), (-255, 255),
                                             dtype=qx.I32)),
         lambda p: p.conv2d(xi, wi, y), conv_ops, 50, dev)
+    xf, wf = (t.to(dev) for t in inputs.conv_case_f32(8, 64, 56, 56, 128, 3, 3, seed=0))
+    yf = torch.empty((8, 128, 56, 56), dtype=torch.float32, device=dev)
+    out["conv_fp32"] = op_times(
+        torch, lambda: qx.Plan(qx.conv_desc(8, 64, 56, 56, 128, 3, 3, 1, 1, (0, 0), (0, 0),
+                                            dtype=qx.F32)),
+        lambda p: p.conv2d(xf, wf, yf), conv_ops, 50, dev)
+    out["conv_fp32"]["workload"] = "x 8x64x56x56, w 128x64x3x3 fp32 N(0,1), 3xTF32"
     Q, Kt, V = (t.to(dev) for t in inputs.attn_case(1024, 64, -7, 7, seed=0))
     O = torch.empty((1024, 64), dtype=torch.int32, device=dev)
     attn_ops = 4.0 * 1024 * 1024 * 64
@@ -241,7 +248,48 @@ def operators(torch, qx, inputs, dev):
     out["attn_int32"] = op_times(
         torch, lambda: qx.Plan(qx.attn_desc(1024, 64, (-7, 7), (-7, 7), (-7, 7), dtype=qx.I32)),
         lambda p: p.attn(Qi, Ki, Vi, O), attn_ops, 50, dev)
+    Qf, Kf, Vf = (t.to(dev) for t in inputs.attn_case_f32(1024, 64, seed=0))
+    Of = torch.empty((1024, 64), dtype=torch.float32, device=dev)
+    out["attn_fp32"] = op_times(
+        torch, lambda: qx.Plan(qx.attn_desc(1024, 64, (0, 0), (0, 0), (0, 0), dtype=qx.F32)),
+        lambda p: p.attn(Qf, Kf, Vf, Of), attn_ops, 50, dev)
+    out["attn_fp32"]["workload"] = "Q,K,V 1024x64 fp32 N(0,1), 3xTF32"
     return out
+
+
+def sweep(args):
+    """Setup / cached / execute-only times of every workload (Table 1 GEMM
+    sizes as INT16 and INT32, the skinny shape, conv, attention, 8192^3), one
+    JSON line each."""
+    import torch
+
+    from paper_2606_09905_gb300 import _build
+    _build.build()
+    from paper_2606_09905_gb300 import inputs, qx
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    rows = []
+    shapes = [(256, 256, 256, 1023), (512, 512, 512, 1023), (768, 768, 768, 1023),
+              (1024, 1024, 1024, 1023), (2048, 2048, 2048, 1023), (4096, 64, 1024, 1023),
+              (8192, 8192, 8192, 500)]
+    for (m, n, k, r) in shapes:
+        for dt, tdt in ((qx.I16, torch.int16), (qx.I32, torch.int32)):
+            if m == 8192 and dt == qx.I32:
+                continue
+            A, B = inputs.gemm_case(m, n, k, -r, r, seed=0, dtype=tdt)
+            A, B = A.to(dev), B.to(dev)
+            C = torch.empty((m, n), dtype=torch.int32, device=dev)
+            fn = "gemm_i16_i32" if dt == qx.I16 else "gemm_i32"
+            res = op_times(torch, lambda: qx.Plan(qx.gemm_desc(m, n, k, (-r, r), (-r, r), dtype=dt)),
+                           lambda p: getattr(p, fn)(A, B, C), 2.0 * m * n * k,
+                           20 if m >= 4096 else 100, dev)
+            res.update(workload=f"gemm {m}x{n}x{k} {'int16' if dt == qx.I16 else 'int32'} [-{r},{r}]")
+            rows.append(res)
+    rows += [dict(v, workload=v.get("workload", k) + f" ({k})") for k, v in
+             operators(torch, qx, inputs, dev).items()]
+    for r in rows:
+        print(json.dumps(r), flush=True)
+    return 0
 
 
 # -------------------------------------------------------------------- main
@@ -446,6 +494,8 @@ def main():
     ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["qx", "reference"], default="qx")
+    ap.add_argument("--sweep", action="store_true",
+                    help="time every workload (setup / cached / execute-only), one JSON line each")
     ap.add_argument("--no-operators", action="store_true", help="skip the conv/attention timings")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
@@ -459,6 +509,8 @@ def main():
         raise SystemExit("--warmup must be at least 3")
     if args.impl == "reference":
         return run_reference(args)
+    if args.sweep:
+        return sweep(args)
     return run_qx(args)
 
 

@@ -31,7 +31,17 @@ bool limb_gemm_supported(int na, int nb);
 int limb_gemm_rows_per_limb(int na);
 cudaError_t limb_gemm_prepare(int na, int nb);
 cudaError_t limb_gemm_launch(int na, int nb, const MmaArgs &a, int grid, cudaStream_t stream);
+cudaError_t tf32x3_prepare();
+cudaError_t tf32x3_launch(const MmaArgs &a, int grid, cudaStream_t stream);
+cudaError_t launch_pack_conv_f32(const float *x, const float *w, int n, int c, int h, int wd,
+                                 int k_out, int r, int s, int Cp, float *x_planes, float *w_planes,
+                                 int num_sms, cudaStream_t st);
 cudaError_t attn_prepare();
+cudaError_t attn_f32_prepare();
+cudaError_t attn_f32_launch(const AttnArgs &a, cudaStream_t stream);
+cudaError_t launch_pack_attn_f32(const float *Q, const float *K, const float *V, int L, int d, int Lp,
+                                 float *q, float *k, float *vt, unsigned *counters, int q_tiles,
+                                 int num_sms, cudaStream_t st);
 cudaError_t attn_launch(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_pack_gemm(bool i32, const void *A, const void *B, int64_t lda, int64_t ldb,
                              int M, int N, int K, int Kp, __half *a_planes, __half *bt_planes,
@@ -94,11 +104,13 @@ struct qx_plan_s {
     MmaArgs mma{};
     int grid = 0;
     __half *planes_n = nullptr, *planes_m = nullptr;
+    float *fplanes_n = nullptr, *fplanes_m = nullptr;   // FP32 kinds
     int Kp = 0, Cp = 0;
     // attention
     AttnArgs attn{};
     int s_shift = 0, max_keys = 0, dp = 0, Lp = 0;
     __half *aq = nullptr, *ak = nullptr, *avt = nullptr;
+    float *fq = nullptr, *fk = nullptr, *fvt = nullptr;   // FP32 kind
 };
 
 // -------------------------------------------------------- TMA descriptors
@@ -127,9 +139,10 @@ static qx_status load_encoders() {
 
 // K-major FP16 tensor of `rank` dims (dims[0] innermost), 128-byte swizzle.
 static qx_status encode_tiled(CUtensorMap *map, const void *base, int rank, const uint64_t *dims,
-                              const uint64_t *strides_bytes, const uint32_t *box) {
+                              const uint64_t *strides_bytes, const uint32_t *box,
+                              CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_FLOAT16) {
     cuuint32_t estr[5] = {1, 1, 1, 1, 1};
-    CUresult r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, rank, const_cast<void *>(base),
+    CUresult r = g_encode_tiled(map, dtype, rank, const_cast<void *>(base),
                                 dims, strides_bytes, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                                 CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -163,9 +176,12 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
     if (!d) return fail(QX_ERR_INVALID_ARG, "null descriptor");
     if (d->in_dtype != QX_I16 && d->in_dtype != QX_I32 && d->in_dtype != QX_F32)
         return fail(QX_ERR_INVALID_ARG, "unknown in_dtype %d", int(d->in_dtype));
-    if (d->in_dtype == QX_F32) return fail(QX_ERR_UNSUPPORTED, "FP32 plans are not available");
+    if (d->in_dtype == QX_F32 && d->op == QX_OP_GEMM)
+        return fail(QX_ERR_UNSUPPORTED, "FP32 plans exist for conv and attention only");
     const bool i16 = d->in_dtype == QX_I16;
+    const bool f32 = d->in_dtype == QX_F32;
     auto range_ok = [&](qx_range r) {
+        if (f32) return true;   // no range contract for FP32 operands
         if (bad_range(r)) return false;
         if (i16) return r.lo >= -32768 && r.hi <= 32767;
         return r.lo >= INT32_MIN && r.hi <= INT32_MAX;
@@ -193,6 +209,22 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
                 return fail(QX_ERR_UNSUPPORTED, "conv pad/filter/stride beyond the im2col path");
             if (!range_ok(d->range_a) || !range_ok(d->range_b))
                 return fail(QX_ERR_INVALID_ARG, "operand range empty or outside the dtype");
+            if (f32) {
+                // 3xTF32: big/small parts of x (M side) and w (N side), one
+                // FP32 accumulator over the whole reduction
+                const int64_t Cp32 = (d->c + kBK32 - 1) / kBK32 * kBK32;
+                Scheme s;
+                s.kind = kKindTf32x3;
+                s.n.limbs = 2;
+                s.m.limbs = 2;
+                s.k = d->r * d->s * Cp32;
+                s.chunk_kb = s.k / kBK32;
+                s.n_chunks = 1;
+                s.acc_bound = 0;
+                out[0] = s;
+                *count = 1;
+                return QX_OK;
+            }
             const int64_t Cp = (d->c + 63) / 64 * 64;
             // N side = weights (output channels), M side = x (output pixels)
             if (!plan_contraction(d->range_b, d->range_a, d->r * d->s * Cp, &out[0]))
@@ -205,6 +237,23 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
             if (d->L < 1 || d->d < 1 || d->L > (1 << 24))
                 return fail(QX_ERR_INVALID_ARG, "attention sizes out of range");
             if (d->d > 128) return fail(QX_ERR_UNSUPPORTED, "attention head size above 128");
+            if (f32) {
+                if (d->d > 64) return fail(QX_ERR_UNSUPPORTED, "FP32 attention head size above 64");
+                Scheme s0, s1;   // 3xTF32 on both products, one FP32 accumulator each
+                s0.kind = s1.kind = kKindTf32x3;
+                s0.n.limbs = s0.m.limbs = 2;
+                s0.k = d->d;
+                s0.chunk_kb = 2;
+                s0.n_chunks = 1;
+                s1.n.limbs = s1.m.limbs = 2;
+                s1.k = d->L;
+                s1.chunk_kb = (d->L + kBK32 - 1) / kBK32;
+                s1.n_chunks = 1;
+                out[0] = s0;
+                out[1] = s1;
+                *count = 2;
+                return QX_OK;
+            }
             if (!range_ok(d->range_a) || !range_ok(d->range_b) || !range_ok(d->range_c))
                 return fail(QX_ERR_INVALID_ARG, "operand range empty or outside the dtype");
             auto mag = [](qx_range r) { return std::max(r.lo < 0 ? -r.lo : r.lo, r.hi < 0 ? -r.hi : r.hi); };
@@ -331,8 +380,73 @@ static qx_status build_gemm(qx_plan p) {
     return QX_OK;
 }
 
+static qx_status build_conv_f32(qx_plan p) {
+    const qx_plan_desc &d = p->desc;
+    const int64_t P = (d.h + 2 * d.pad - d.r) / d.stride + 1;
+    const int64_t Q = (d.w + 2 * d.pad - d.s) / d.stride + 1;
+    p->Cp = int((d.c + kBK32 - 1) / kBK32 * kBK32);
+    const size_t x_bytes = size_t(2) * d.n * d.h * d.w * p->Cp * 4;
+    const size_t w_bytes = size_t(2) * d.k_out * d.r * d.s * p->Cp * 4;
+    p->ws_bytes = 256 + align256(x_bytes) + align256(w_bytes);
+    QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
+    p->err = static_cast<int *>(p->ws);
+    p->fplanes_m = reinterpret_cast<float *>(static_cast<char *>(p->ws) + 256);
+    p->fplanes_n = reinterpret_cast<float *>(static_cast<char *>(p->ws) + 256 + align256(x_bytes));
+    QX_CUDA(cudaMemset(p->err, 0, sizeof(int)), "error word reset");
+
+    MmaArgs &a = p->mma;
+    memset(&a, 0, sizeof a);
+    for (int j = 0; j < 2; ++j) {
+        const cuuint64_t dims[4] = {cuuint64_t(p->Cp), cuuint64_t(d.w), cuuint64_t(d.h),
+                                    cuuint64_t(d.n)};
+        const cuuint64_t str[3] = {cuuint64_t(p->Cp) * 4, cuuint64_t(d.w) * p->Cp * 4,
+                                   cuuint64_t(d.h) * d.w * p->Cp * 4};
+        const int lower[2] = {int(-d.pad), int(-d.pad)};
+        const int upper[2] = {int(d.pad - (d.s - 1)), int(d.pad - (d.r - 1))};
+        const cuuint32_t estr[4] = {1, cuuint32_t(d.stride), cuuint32_t(d.stride), 1};
+        CUresult r = g_encode_im2col(&a.tm_m[j], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4,
+                                     p->fplanes_m + size_t(j) * d.n * d.h * d.w * p->Cp, dims, str,
+                                     lower, upper, kBK32, kBM, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS)
+            return fail(QX_ERR_UNSUPPORTED, "cuTensorMapEncodeIm2col failed (%d)", int(r));
+    }
+    const int64_t Kg = d.r * d.s * p->Cp;
+    {
+        const uint64_t dims[3] = {uint64_t(Kg), uint64_t(d.k_out), 2};
+        const uint64_t str[2] = {uint64_t(Kg) * 4, uint64_t(d.k_out) * Kg * 4};
+        const uint32_t box[3] = {kBK32, 128, 2};
+        qx_status st = encode_tiled(&a.tm_n, p->fplanes_n, 3, dims, str, box,
+                                    CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
+        if (st != QX_OK) return st;
+    }
+    a.err = p->err;
+    a.out_row_stride = P * Q;
+    a.mode = 1;
+    a.m_extent = int(d.n * P * Q);
+    a.n_extent = int(d.k_out);
+    a.kblocks = int(Kg / kBK32);
+    a.chunk_kb = a.kblocks;
+    a.tiles_m = int((a.m_extent + kBM - 1) / kBM);
+    a.tiles_n = int((d.k_out + 127) / 128);
+    a.group_n = std::max(1, std::min(16, a.tiles_n));
+    a.c_blocks = p->Cp / kBK32;
+    a.S = int(d.s);
+    a.Q = int(Q);
+    a.PQ = int(P * Q);
+    a.stride = int(d.stride);
+    a.pad = int(d.pad);
+    a.k_out = int(d.k_out);
+    const int tiles = a.tiles_m * a.tiles_n;
+    p->grid = std::max(1, std::min(tiles, p->num_sms));
+    QX_CUDA(tf32x3_prepare(), "kernel attributes");
+    return QX_OK;
+}
+
 static qx_status build_conv(qx_plan p) {
     const qx_plan_desc &d = p->desc;
+    if (d.in_dtype == QX_F32) return build_conv_f32(p);
     const Scheme &s = p->scheme[0];
     const int nw = s.n.limbs, nx = s.m.limbs;
     const int mr = limb_gemm_rows_per_limb(nw);
@@ -399,8 +513,66 @@ static qx_status build_conv(qx_plan p) {
     return QX_OK;
 }
 
+static qx_status build_attn_f32(qx_plan p) {
+    const qx_plan_desc &d = p->desc;
+    p->dp = 64;
+    p->Lp = int((d.L + 7) / 8 * 8);
+    AttnArgs &a = p->attn;
+    memset(&a, 0, sizeof a);
+    a.L = int(d.L);
+    a.d = int(d.d);
+    a.q_tiles = int((d.L + 127) / 128);
+    const int key_blocks = int((d.L + 31) / 32);
+    int splits = std::max(1, std::min(key_blocks, (p->num_sms + a.q_tiles - 1) / a.q_tiles));
+    const int per = (key_blocks + splits - 1) / splits;
+    splits = (key_blocks + per - 1) / per;
+    a.key_splits = splits;
+    a.keys_per_split = per * 32;
+    const size_t qk_bytes = size_t(2) * d.L * 64 * 4;
+    const size_t vt_bytes = size_t(2) * 64 * p->Lp * 4;
+    const size_t part_bytes = size_t(a.q_tiles) * splits * 128 * 64 * 4;
+    const size_t cnt_bytes = size_t(a.q_tiles) * 4;
+    p->ws_bytes = 256 + 2 * align256(qk_bytes) + align256(vt_bytes) + align256(part_bytes) +
+                  align256(cnt_bytes);
+    QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
+    char *base = static_cast<char *>(p->ws);
+    p->err = reinterpret_cast<int *>(base);
+    size_t off = 256;
+    p->fq = reinterpret_cast<float *>(base + off);
+    off += align256(qk_bytes);
+    p->fk = reinterpret_cast<float *>(base + off);
+    off += align256(qk_bytes);
+    p->fvt = reinterpret_cast<float *>(base + off);
+    off += align256(vt_bytes);
+    a.partial = reinterpret_cast<float *>(base + off);
+    off += align256(part_bytes);
+    a.counters = reinterpret_cast<unsigned *>(base + off);
+    QX_CUDA(cudaMemset(p->ws, 0, p->ws_bytes), "workspace reset");
+    {
+        const uint64_t dims[3] = {64, uint64_t(d.L), 2};
+        const uint64_t str[2] = {64 * 4, uint64_t(d.L) * 64 * 4};
+        const uint32_t boxq[3] = {32, 128, 2};
+        const uint32_t boxk[3] = {32, 32, 2};
+        qx_status st = encode_tiled(&a.tm_q, p->fq, 3, dims, str, boxq, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
+        if (st != QX_OK) return st;
+        st = encode_tiled(&a.tm_k, p->fk, 3, dims, str, boxk, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
+        if (st != QX_OK) return st;
+    }
+    {
+        const uint64_t dims[3] = {uint64_t(d.L), 64, 2};
+        const uint64_t str[2] = {uint64_t(p->Lp) * 4, uint64_t(64) * p->Lp * 4};
+        const uint32_t box[3] = {32, 128, 2};
+        qx_status st = encode_tiled(&a.tm_vt, p->fvt, 3, dims, str, box, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
+        if (st != QX_OK) return st;
+    }
+    a.err = p->err;
+    QX_CUDA(attn_f32_prepare(), "kernel attributes");
+    return QX_OK;
+}
+
 static qx_status build_attn(qx_plan p) {
     const qx_plan_desc &d = p->desc;
+    if (d.in_dtype == QX_F32) return build_attn_f32(p);
     p->dp = d.d <= 64 ? 64 : 128;
     p->Lp = int((d.L + 7) / 8 * 8);
     const size_t qk_bytes = size_t(d.L) * p->dp * 2;
@@ -597,6 +769,14 @@ static qx_status pack(qx_plan p, const void *a, const void *b, const void *c, cu
             if (!a || !b) return fail(QX_ERR_INVALID_ARG, "null operand");
             if (!aligned16(a) || !aligned16(b))
                 return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+            if (d.in_dtype == QX_F32) {
+                QX_CUDA(launch_pack_conv_f32(static_cast<const float *>(a),
+                                             static_cast<const float *>(b), int(d.n), int(d.c),
+                                             int(d.h), int(d.w), int(d.k_out), int(d.r), int(d.s),
+                                             p->Cp, p->fplanes_m, p->fplanes_n, p->num_sms, st),
+                        "operand packing launch");
+                return QX_OK;
+            }
             const Scheme &s = p->scheme[0];
             QX_CUDA(launch_pack_conv(i32, a, b, int(d.n), int(d.c), int(d.h), int(d.w),
                                      int(d.k_out), int(d.r), int(d.s), p->Cp, p->planes_m,
@@ -609,6 +789,15 @@ static qx_status pack(qx_plan p, const void *a, const void *b, const void *c, cu
             if (!a || !b || !c) return fail(QX_ERR_INVALID_ARG, "null operand");
             if (!aligned16(a) || !aligned16(b) || !aligned16(c))
                 return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+            if (d.in_dtype == QX_F32) {
+                QX_CUDA(launch_pack_attn_f32(static_cast<const float *>(a),
+                                             static_cast<const float *>(b),
+                                             static_cast<const float *>(c), int(d.L), int(d.d),
+                                             p->Lp, p->fq, p->fk, p->fvt, p->attn.counters,
+                                             p->attn.q_tiles, p->num_sms, st),
+                        "operand packing launch");
+                return QX_OK;
+            }
             QX_CUDA(launch_pack_attn(i32, a, b, c, int(d.L), int(d.d), p->dp, p->Lp, p->aq, p->ak,
                                      p->avt, check, d.range_a, d.range_b, d.range_c, p->err,
                                      p->num_sms, st),
@@ -640,15 +829,22 @@ static qx_status run_packed(qx_plan p, void *out, cudaStream_t st) {
         }
         case QX_OP_CONV2D: {
             MmaArgs a = p->mma;
-            a.out = static_cast<int32_t *>(out);
-            QX_CUDA(limb_gemm_launch(p->scheme[0].n.limbs, p->scheme[0].m.limbs, a, p->grid, st),
-                    "conv launch");
+            a.out = out;
+            if (d.in_dtype == QX_F32)
+                QX_CUDA(tf32x3_launch(a, p->grid, st), "conv launch");
+            else
+                QX_CUDA(limb_gemm_launch(p->scheme[0].n.limbs, p->scheme[0].m.limbs, a, p->grid, st),
+                        "conv launch");
             return QX_OK;
         }
         case QX_OP_ATTN: {
-            QX_CUDA(cudaMemsetAsync(out, 0, size_t(d.L) * d.d * 4, st), "zero output");
             AttnArgs a = p->attn;
-            a.out = static_cast<int32_t *>(out);
+            a.out = out;
+            if (d.in_dtype == QX_F32) {
+                QX_CUDA(attn_f32_launch(a, st), "attention launch");
+                return QX_OK;
+            }
+            QX_CUDA(cudaMemsetAsync(out, 0, size_t(d.L) * d.d * 4, st), "zero output");
             QX_CUDA(attn_launch(a, st), "attention launch");
             return QX_OK;
         }

@@ -226,6 +226,21 @@ __device__ __forceinline__ void tmem_wait_ld(uint32_t (&v)[32]) {
                  : "memory");
 }
 
+// --------------------------------------------------------------- TF32 split
+// x rounded to TF32 (10 explicit mantissa bits, round to nearest, ties away).
+__device__ __forceinline__ float tf32_round(float x) {
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+    return __uint_as_float(r);
+}
+
+// x = big + small with both parts TF32 values: big keeps the top 11
+// significant bits, small the next 11 (the residual x - big is exact in FP32).
+__device__ __forceinline__ void tf32_split(float x, float &big, float &small) {
+    big = tf32_round(x);
+    small = tf32_round(x - big);
+}
+
 // ------------------------------------------------------------- limb digits
 // Balanced base-2^s digits of x: digit i in [-2^(s-1), 2^(s-1)) for i < NL-1,
 // the top digit takes what remains; x = sum_i digit_i * 2^(i*s).

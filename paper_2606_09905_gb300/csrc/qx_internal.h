@@ -14,8 +14,14 @@ namespace qx {
 constexpr int64_t kAccLimit = int64_t(1) << 24;
 // Largest |integer| an FP16 limb may hold exactly (11-bit significand).
 constexpr int64_t kHalfExact = 2048;
-// K extent of one pipeline stage: 64 FP16 values = one 128-byte swizzle row.
+// K extent of one pipeline stage: 64 FP16 values = one 128-byte swizzle row
+// (32 values for the TF32 kind, whose elements take 4 bytes).
 constexpr int kBK = 64;
+constexpr int kBK32 = 32;
+
+// Operand kinds of the tiled kernel.
+constexpr int kKindExact = 0;   // FP16 integer digits, exact int32 result
+constexpr int kKindTf32x3 = 1;  // FP32 operands as TF32 big + small parts
 // Rows of the tile on the MMA's M side (TMEM lanes).
 constexpr int kBM = 128;
 
@@ -39,13 +45,14 @@ struct Scheme {
     int64_t chunk_kb = 1;   // k-blocks (of kBK) per FP32 chunk
     int64_t n_chunks = 0;
     int64_t acc_bound = 0;  // max |partial| an accumulator can reach in a chunk
+    int kind = kKindExact;  // kKindTf32x3: FP32 operands, chunk_kb counts 32-wide k-blocks
 };
 
 // Kernel arguments of the tiled limb GEMM, cached in the plan.
 struct MmaArgs {
     CUtensorMap tm_m[2];      // M-side operand, one map per limb
     CUtensorMap tm_n;         // N-side operand: 3-D (k, row, limb)
-    int32_t *out;             // set per call
+    void *out;                // set per call: int32 (exact integer kinds) or float (TF32x3)
     int *err;                 // device error word
     int64_t out_row_stride;   // elements between consecutive N-side rows
     int mode;                 // 0 = GEMM, 1 = conv (im2col M side, NCHW out)
@@ -61,15 +68,19 @@ struct MmaArgs {
 
 // Kernel arguments of the fused attention core.
 struct AttnArgs {
-    CUtensorMap tm_q;         // Q   (L x d) fp16, 2-D
-    CUtensorMap tm_k;         // K   (L x d) fp16, 2-D
-    CUtensorMap tm_vt;        // V^T (d x L) fp16, 2-D (K-major for the 2nd MMA)
-    int32_t *out;             // O (L x d) int32, zeroed before the launch
+    CUtensorMap tm_q;         // Q   (L x d): fp16 2-D, or fp32 3-D (d, L, big/small)
+    CUtensorMap tm_k;         // K   (L x d): same
+    CUtensorMap tm_vt;        // V^T (d x L): fp16 2-D, or fp32 3-D (L, d, big/small)
+    void *out;                // O (L x d): int32 (zeroed before the launch) or float
     int *err;
     int L, d;
     int q_tiles, key_splits, keys_per_split;
-    int s_shift;              // digit width of the S limbs
+    int s_shift;              // digit width of the S limbs (integer kind)
     int o_chunk_kb;           // key-blocks per FP32 chunk of the second product
+    // FP32 kind: per-CTA partial O (q_tiles x key_splits x 128 x 64 floats) and
+    // one arrival counter per query tile (zero between calls)
+    float *partial;
+    unsigned *counters;
 };
 
 }  // namespace qx

@@ -25,6 +25,13 @@
 //               of the N-side rows; running int32 sums live in registers.
 // Accumulators are double-buffered in TMEM whenever they fit in 256 columns,
 // so the epilogue drains chunk c while the tensor cores run chunk c + 1.
+//
+// FP32 kind (Table 2 FP32 conv row).  The same pipeline runs kind::tf32 with
+// FP32 operands split as x = x_big + x_small (both TF32-rounded): each k-step
+// issues x_big * [w_big; w_small] (N = 256) and x_small * w_big (N = 128) into
+// one FP32 accumulator, and the epilogue adds its two column halves -- three
+// of the four cross products ("3xTF32"), error about 3 * 2^-22 relative per
+// product, far inside the 1e-5 * sum|a||b| tolerance.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -33,8 +40,9 @@
 
 namespace qx {
 
-template <int NA, int NB>
+template <int NA, int NB, int KIND>
 struct TileCfg {
+    static constexpr bool TF = KIND == kKindTf32x3;
     static constexpr int MR = NA <= 2 ? 128 : 64;   // N-side rows per limb
     static constexpr int UN = NA * MR;              // MMA N
     static constexpr int M_TILE = kBM * 128;        // bytes of one M-side limb tile
@@ -42,7 +50,9 @@ struct TileCfg {
     static constexpr int STAGE = NB * M_TILE + N_TILE;
     static constexpr int STAGES_FIT = (200 * 1024) / STAGE;
     static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
-    static constexpr int ACC_COLS = NB * UN;        // TMEM columns per accumulator set
+    // TMEM columns per accumulator set: every M-side limb has its own for the
+    // exact kind; the TF32 kind sums all products into one.
+    static constexpr int ACC_COLS = TF ? UN : NB * UN;
     static constexpr int NBUF = ACC_COLS <= 256 ? 2 : 1;
     static constexpr int TMEM_NEED = ACC_COLS * NBUF;
     static constexpr int TMEM_COLS = TMEM_NEED <= 32    ? 32
@@ -51,13 +61,17 @@ struct TileCfg {
                                      : TMEM_NEED <= 256 ? 256
                                                         : 512;
     static constexpr int RPT = MR / 2;              // N-side rows per epilogue thread
-    static constexpr uint32_t IDESC = make_idesc(kBM, UN, 0);
+    static constexpr uint32_t AB_TYPE = TF ? 2u : 0u;
+    static constexpr uint32_t IDESC = make_idesc(kBM, UN, AB_TYPE);
+    static constexpr uint32_t IDESC_FIRST = make_idesc(kBM, MR, AB_TYPE);  // first N-side limb only
+    static constexpr int BK_ELEMS = TF ? kBK32 : kBK;                     // K per 128-byte row
     static constexpr int BAR_BYTES = 256;
     static constexpr int SMEM = STAGES * STAGE + BAR_BYTES + 1024;
     static constexpr int THREADS = 320;
     static_assert(UN % 16 == 0 && UN >= 16 && UN <= 256, "MMA N out of range");
     static_assert(TMEM_NEED <= 512, "accumulators exceed tensor memory");
     static_assert(RPT % 32 == 0, "epilogue works in 32-column TMEM loads");
+    static_assert(!TF || (NA == 2 && NB == 2), "TF32x3 stacks big/small on both sides");
 };
 
 // Tile order: groups of `group_n` N-side tiles, M-side tiles inside a group,
@@ -72,9 +86,9 @@ __device__ __forceinline__ void tile_coords(int t, const MmaArgs &a, int &tm, in
     tm = r / gs;
 }
 
-template <int NA, int NB>
+template <int NA, int NB, int KIND>
 __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant__ MmaArgs a) {
-    using T = TileCfg<NA, NB>;
+    using T = TileCfg<NA, NB, KIND>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -143,8 +157,8 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
                     if (a.mode == 0) {
 #pragma unroll
                         for (int j = 0; j < NB; ++j)
-                            tma_load_2d(st + j * T::M_TILE, &a.tm_m[j], &full[stage], kb * kBK,
-                                        tm * kBM);
+                            tma_load_2d(st + j * T::M_TILE, &a.tm_m[j], &full[stage],
+                                        kb * T::BK_ELEMS, tm * kBM);
                     } else {
                         const int tap = kb / a.c_blocks;
                         const int cb = kb - tap * a.c_blocks;
@@ -153,11 +167,11 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
 #pragma unroll
                         for (int j = 0; j < NB; ++j)
                             tma_load_im2col_4d(st + j * T::M_TILE, &a.tm_m[j], &full[stage],
-                                               cb * kBK, ow * a.stride - a.pad,
+                                               cb * T::BK_ELEMS, ow * a.stride - a.pad,
                                                oh * a.stride - a.pad, img, uint16_t(s),
                                                uint16_t(r));
                     }
-                    tma_load_3d(st + NB * T::M_TILE, &a.tm_n, &full[stage], kb * kBK,
+                    tma_load_3d(st + NB * T::M_TILE, &a.tm_n, &full[stage], kb * T::BK_ELEMS,
                                 tn * T::MR, 0);
                     ++issued;
                     if (++stage == T::STAGES) {
@@ -212,13 +226,21 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
                         tc_fence_after();
                         const uint32_t sbase = smem_addr(smem + stage * T::STAGE);
 #pragma unroll
-                        for (int kk = 0; kk < kBK / 16; ++kk) {
+                        for (int kk = 0; kk < 4; ++kk) {          // 4 x 32 bytes of K per row
                             const uint64_t bdesc = make_sdesc(sbase + NB * T::M_TILE + kk * 32);
+                            const uint32_t acc = (kb > kb0 || kk > 0) ? 1u : 0u;
+                            if constexpr (T::TF) {
+                                // x_big * [w_big; w_small], then x_small * w_big
+                                mma_tf32(d0, make_sdesc(sbase + kk * 32), bdesc, T::IDESC, acc);
+                                mma_tf32(d0, make_sdesc(sbase + T::M_TILE + kk * 32), bdesc,
+                                         T::IDESC_FIRST, 1u);
+                            } else {
 #pragma unroll
-                            for (int j = 0; j < NB; ++j) {
-                                const uint64_t adesc = make_sdesc(sbase + j * T::M_TILE + kk * 32);
-                                mma_f16(d0 + j * T::UN, adesc, bdesc, T::IDESC,
-                                        (kb > kb0 || kk > 0) ? 1u : 0u);
+                                for (int j = 0; j < NB; ++j) {
+                                    const uint64_t adesc =
+                                        make_sdesc(sbase + j * T::M_TILE + kk * 32);
+                                    mma_f16(d0 + j * T::UN, adesc, bdesc, T::IDESC, acc);
+                                }
                             }
                         }
                         tc_commit(&empty[stage]);
@@ -247,6 +269,7 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
         for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
             int tm, tn;
             tile_coords(t, a, tm, tn);
+            // running sums: wrapping int32 (exact kind) or FP32 (TF32 kind)
             uint32_t acc[T::RPT];
 #pragma unroll
             for (int r = 0; r < T::RPT; ++r) acc[r] = 0u;
@@ -260,20 +283,36 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
                 tc_fence_after();
                 const uint32_t tb =
                     tmem_base + (uint32_t(q * 32) << 16) + buf * T::ACC_COLS + hh * T::RPT;
+                if constexpr (T::TF) {
 #pragma unroll
-                for (int j = 0; j < NB; ++j) {
+                    for (int p = 0; p < T::RPT / 32; ++p) {
+                        uint32_t v0[32], v1[32];
+                        tmem_ld32(tb + p * 32, v0);              // x_big*w_big + x_small*w_big
+                        tmem_ld32(tb + T::MR + p * 32, v1);      // x_big*w_small
+                        tmem_wait_ld(v0);
+                        tmem_wait_ld(v1);
 #pragma unroll
-                    for (int i = 0; i < NA; ++i) {
-                        const int sh = i * a.shift_n + j * a.shift_m;
+                        for (int x = 0; x < 32; ++x)
+                            acc[p * 32 + x] = __float_as_uint(
+                                __uint_as_float(acc[p * 32 + x]) +
+                                (__uint_as_float(v0[x]) + __uint_as_float(v1[x])));
+                    }
+                } else {
 #pragma unroll
-                        for (int p = 0; p < T::RPT / 32; ++p) {
-                            uint32_t v[32];
-                            tmem_ld32(tb + j * T::UN + i * T::MR + p * 32, v);
-                            tmem_wait_ld(v);
+                    for (int j = 0; j < NB; ++j) {
 #pragma unroll
-                            for (int x = 0; x < 32; ++x)
-                                acc[p * 32 + x] +=
-                                    uint32_t(__float2int_rn(__uint_as_float(v[x]))) << sh;
+                        for (int i = 0; i < NA; ++i) {
+                            const int sh = i * a.shift_n + j * a.shift_m;
+#pragma unroll
+                            for (int p = 0; p < T::RPT / 32; ++p) {
+                                uint32_t v[32];
+                                tmem_ld32(tb + j * T::UN + i * T::MR + p * 32, v);
+                                tmem_wait_ld(v);
+#pragma unroll
+                                for (int x = 0; x < 32; ++x)
+                                    acc[p * 32 + x] +=
+                                        uint32_t(__float2int_rn(__uint_as_float(v[x]))) << sh;
+                            }
                         }
                     }
                 }
@@ -291,11 +330,11 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
                 lane_off = int64_t(img) * a.k_out * a.PQ + (mrow - img * a.PQ);
             }
             const int nrow0 = tn * T::MR + hh * T::RPT;
-            int32_t *o = a.out + lane_off + int64_t(nrow0) * a.out_row_stride;
+            // both output types are 32-bit: store the raw words
+            uint32_t *o = static_cast<uint32_t *>(a.out) + lane_off + int64_t(nrow0) * a.out_row_stride;
 #pragma unroll
             for (int r = 0; r < T::RPT; ++r) {
-                if (lane_ok && nrow0 + r < a.n_extent)
-                    o[int64_t(r) * a.out_row_stride] = int32_t(acc[r]);
+                if (lane_ok && nrow0 + r < a.n_extent) o[int64_t(r) * a.out_row_stride] = acc[r];
             }
         }
     }
@@ -309,15 +348,17 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
 }
 
 // ------------------------------------------------------------------- host
-template <int NA, int NB>
+template <int NA, int NB, int KIND = kKindExact>
 static cudaError_t prepare_t() {
-    return cudaFuncSetAttribute(limb_gemm_kernel<NA, NB>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, TileCfg<NA, NB>::SMEM);
+    return cudaFuncSetAttribute(limb_gemm_kernel<NA, NB, KIND>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                TileCfg<NA, NB, KIND>::SMEM);
 }
 
-template <int NA, int NB>
+template <int NA, int NB, int KIND = kKindExact>
 static cudaError_t launch_t(const MmaArgs &a, int grid, cudaStream_t stream) {
-    limb_gemm_kernel<NA, NB><<<grid, TileCfg<NA, NB>::THREADS, TileCfg<NA, NB>::SMEM, stream>>>(a);
+    using T = TileCfg<NA, NB, KIND>;
+    limb_gemm_kernel<NA, NB, KIND><<<grid, T::THREADS, T::SMEM, stream>>>(a);
     return cudaGetLastError();
 }
 
@@ -346,6 +387,12 @@ cudaError_t limb_gemm_prepare(int na, int nb) { QX_LIMB_DISPATCH(prepare_t) }
 
 cudaError_t limb_gemm_launch(int na, int nb, const MmaArgs &a, int grid, cudaStream_t stream) {
     QX_LIMB_DISPATCH(launch_t, a, grid, stream)
+}
+
+cudaError_t tf32x3_prepare() { return prepare_t<2, 2, kKindTf32x3>(); }
+
+cudaError_t tf32x3_launch(const MmaArgs &a, int grid, cudaStream_t stream) {
+    return launch_t<2, 2, kKindTf32x3>(a, grid, stream);
 }
 
 }  // namespace qx

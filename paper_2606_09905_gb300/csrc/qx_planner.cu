@@ -124,8 +124,9 @@ void scheme_to_info(const Scheme &s, qx_scheme_info *o) {
     o->shift_a = s.n.shift;
     o->limbs_b = s.m.limbs;
     o->shift_b = s.m.shift;
-    o->mma_per_kstep = s.n.limbs * s.m.limbs;
-    o->chunk_k = s.chunk_kb * kBK;
+    const bool tf = s.kind == kKindTf32x3;
+    o->mma_per_kstep = tf ? 3 : s.n.limbs * s.m.limbs;   // 3xTF32 skips small * small
+    o->chunk_k = s.chunk_kb * (tf ? kBK32 : kBK);
     o->n_chunks = s.n_chunks;
     o->acc_bound = s.acc_bound;
     o->k = s.k;

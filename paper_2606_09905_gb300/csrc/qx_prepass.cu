@@ -204,6 +204,77 @@ __global__ void __launch_bounds__(256) pack_conv_kernel(const ConvPackArgs p) {
     }
 }
 
+// -------------------------------------------------------- conv, FP32 kind
+// x (NCHW float) -> big and small TF32 planes, NHWC, channels padded to Cp
+// (a multiple of 32, one 128-byte row); w (KCRS) -> (k, r, s, Cp) planes.
+struct ConvPackF32Args {
+    const float *x, *w;
+    int n, c, h, wd, k_out, r, s, Cp;
+    float *x_planes;       // [2][n][h][w][Cp]
+    float *w_planes;       // [2][k_out][r][s][Cp]
+    int x_blocks, x_tiles_hw, x_tiles_c;
+};
+
+__device__ __forceinline__ void store_split8(float *plane0, int64_t plane_stride, const float (&v)[8]) {
+    __align__(16) float big[8], small[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) tf32_split(v[e], big[e], small[e]);
+    uint4 *b = reinterpret_cast<uint4 *>(plane0);
+    uint4 *sm = reinterpret_cast<uint4 *>(plane0 + plane_stride);
+    b[0] = reinterpret_cast<uint4 *>(big)[0];
+    b[1] = reinterpret_cast<uint4 *>(big)[1];
+    sm[0] = reinterpret_cast<uint4 *>(small)[0];
+    sm[1] = reinterpret_cast<uint4 *>(small)[1];
+}
+
+__global__ void __launch_bounds__(256) pack_conv_f32_kernel(const ConvPackF32Args p) {
+    __shared__ float tile[64][65];
+    const int HW = p.h * p.wd;
+    if (int(blockIdx.x) < p.x_blocks) {
+        int t = blockIdx.x;
+        const int tc = t % p.x_tiles_c;
+        t /= p.x_tiles_c;
+        const int thw = t % p.x_tiles_hw;
+        const int img = t / p.x_tiles_hw;
+        const int c0 = tc * 64, hw0 = thw * 64;
+        for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
+            const int cr = i >> 6, pc = i & 63;
+            float v = 0.f;
+            if (c0 + cr < p.c && hw0 + pc < HW) v = p.x[(int64_t(img) * p.c + c0 + cr) * HW + hw0 + pc];
+            tile[cr][pc] = v;
+        }
+        __syncthreads();
+        const int64_t plane_stride = int64_t(p.n) * HW * p.Cp;
+        for (int i = threadIdx.x; i < 64 * 8; i += blockDim.x) {
+            const int pr = i >> 3, cg = i & 7;
+            if (hw0 + pr >= HW || c0 + cg * 8 >= p.Cp) continue;
+            float v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = tile[cg * 8 + e][pr];
+            store_split8(p.x_planes + (int64_t(img) * HW + hw0 + pr) * p.Cp + c0 + cg * 8,
+                         plane_stride, v);
+        }
+        return;
+    }
+    const int RS = p.r * p.s;
+    const int cgs = p.Cp >> 3;
+    const int64_t items = int64_t(p.k_out) * RS * cgs;
+    const int64_t plane_stride = int64_t(p.k_out) * RS * p.Cp;
+    for (int64_t it = int64_t(blockIdx.x - p.x_blocks) * blockDim.x + threadIdx.x; it < items;
+         it += int64_t(gridDim.x - p.x_blocks) * blockDim.x) {
+        const int cg = int(it % cgs);
+        const int tap = int((it / cgs) % RS);
+        const int o = int(it / (int64_t(cgs) * RS));
+        float v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int c = cg * 8 + e;
+            v[e] = c < p.c ? p.w[(int64_t(o) * p.c + c) * RS + tap] : 0.f;
+        }
+        store_split8(p.w_planes + (int64_t(o) * RS + tap) * p.Cp + cg * 8, plane_stride, v);
+    }
+}
+
 // ------------------------------------------------------- attention operands
 struct AttnPackArgs {
     const void *Q, *K, *V;
@@ -267,6 +338,57 @@ __global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
 #pragma unroll
         for (int e = 0; e < 8; ++e) v[e] = tile[lg * 8 + e][cr];
         store_limbs8<1>(p.vt + int64_t(c) * p.Lp + l, 0, v, 0);
+    }
+}
+
+// ------------------------------------------------ attention, FP32 kind
+// Q, K (L x d) -> big/small TF32 planes [2][L][64] (zero columns beyond d);
+// V -> V^T planes [2][64][Lp]; the per-query-tile arrival counters of the
+// attention kernel are zeroed here, before every launch.
+struct AttnPackF32Args {
+    const float *Q, *K, *V;
+    int L, d, Lp;
+    float *q, *k, *vt;
+    unsigned *counters;
+    int q_tiles;
+    int qk_blocks, v_tiles_l;
+};
+
+__global__ void __launch_bounds__(256) pack_attn_f32_kernel(const AttnPackF32Args p) {
+    __shared__ float tile[64][65];
+    if (int(blockIdx.x) < p.qk_blocks) {
+        if (blockIdx.x == 0)
+            for (int i = threadIdx.x; i < p.q_tiles; i += blockDim.x) p.counters[i] = 0u;
+        const int64_t items = int64_t(2) * p.L * 8;            // 8 groups of 8 columns
+        for (int64_t it = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; it < items;
+             it += int64_t(p.qk_blocks) * blockDim.x) {
+            const int which = int(it / (int64_t(p.L) * 8));
+            const int64_t rem = it - int64_t(which) * p.L * 8;
+            const int row = int(rem / 8);
+            const int c = int(rem % 8) * 8;
+            const float *src = (which ? p.K : p.Q) + int64_t(row) * p.d;
+            float v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = c + e < p.d ? src[c + e] : 0.f;
+            store_split8((which ? p.k : p.q) + int64_t(row) * 64 + c, int64_t(p.L) * 64, v);
+        }
+        return;
+    }
+    const int t = int(blockIdx.x) - p.qk_blocks;
+    const int l0 = t * 64;
+    for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
+        const int lr = i >> 6, cc = i & 63;
+        tile[lr][cc] = (l0 + lr < p.L && cc < p.d) ? p.V[int64_t(l0 + lr) * p.d + cc] : 0.f;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < 64 * 8; i += blockDim.x) {
+        const int cr = i >> 3, lg = i & 7;
+        const int l = l0 + lg * 8;
+        if (l >= p.Lp) continue;
+        float v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = tile[lg * 8 + e][cr];
+        store_split8(p.vt + int64_t(cr) * p.Lp + l, int64_t(64) * p.Lp, v);
     }
 }
 
@@ -363,6 +485,33 @@ cudaError_t launch_pack_conv(bool i32, const void *x, const void *w, int n, int 
     return i32 ? pack_conv_t<int32_t>(nx, nw, p, grid, st) : pack_conv_t<int16_t>(nx, nw, p, grid, st);
 }
 
+cudaError_t launch_pack_conv_f32(const float *x, const float *w, int n, int c, int h, int wd,
+                                 int k_out, int r, int s, int Cp, float *x_planes, float *w_planes,
+                                 int num_sms, cudaStream_t st) {
+    ConvPackF32Args p;
+    p.x = x;
+    p.w = w;
+    p.n = n;
+    p.c = c;
+    p.h = h;
+    p.wd = wd;
+    p.k_out = k_out;
+    p.r = r;
+    p.s = s;
+    p.Cp = Cp;
+    p.x_planes = x_planes;
+    p.w_planes = w_planes;
+    p.x_tiles_hw = (h * wd + 63) / 64;
+    p.x_tiles_c = (Cp + 63) / 64;
+    p.x_blocks = n * p.x_tiles_hw * p.x_tiles_c;
+    const int64_t w_items = int64_t(k_out) * r * s * (Cp / 8);
+    int w_blocks = int((w_items + 255) / 256);
+    if (w_blocks > num_sms) w_blocks = num_sms;
+    if (w_blocks < 1) w_blocks = 1;
+    pack_conv_f32_kernel<<<p.x_blocks + w_blocks, 256, 0, st>>>(p);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int L, int d,
                              int dp, int Lp, __half *q, __half *k, __half *vt, int check,
                              qx_range rq, qx_range rk, qx_range rv, int *err, int num_sms,
@@ -393,4 +542,30 @@ cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void 
     return cudaGetLastError();
 }
 
+}  // namespace qx
+
+namespace qx {
+cudaError_t launch_pack_attn_f32(const float *Q, const float *K, const float *V, int L, int d, int Lp,
+                                 float *q, float *k, float *vt, unsigned *counters, int q_tiles,
+                                 int num_sms, cudaStream_t st) {
+    AttnPackF32Args p;
+    p.Q = Q;
+    p.K = K;
+    p.V = V;
+    p.L = L;
+    p.d = d;
+    p.Lp = Lp;
+    p.q = q;
+    p.k = k;
+    p.vt = vt;
+    p.counters = counters;
+    p.q_tiles = q_tiles;
+    const int64_t items = int64_t(2) * L * 8;
+    int64_t blocks = (items + 255) / 256;
+    if (blocks > num_sms) blocks = num_sms;
+    p.qk_blocks = int(blocks < 1 ? 1 : blocks);
+    p.v_tiles_l = (Lp + 63) / 64;
+    pack_attn_f32_kernel<<<p.qk_blocks + p.v_tiles_l, 256, 0, st>>>(p);
+    return cudaGetLastError();
+}
 }  // namespace qx

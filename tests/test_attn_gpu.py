@@ -75,3 +75,50 @@ def test_attn_identity_reassociation():
     assert st == qx.OK
     q, k, v = (t.numpy().astype(np.int64) for t in (Q, K, V))
     assert_exact(got, q @ (k.T @ v), f"reassociation {info}")
+
+
+# ------------------------------------------------------------ FP32 (3xTF32)
+def attn_gpu_f32(Q, K, V):
+    L, d = Q.shape
+    with qx.Plan(qx.attn_desc(L, d, (0, 0), (0, 0), (0, 0), dtype=qx.F32)) as plan:
+        O = plan.attn(Q.cuda(), K.cuda(), V.cuda())
+        torch.cuda.synchronize()
+        st = plan.status()
+    return O.cpu().numpy().astype(np.float64), st
+
+
+def within_tolerance(got, Q, K, V, what):
+    """max |err| <= 1e-5 * ((|Q||K|^T)|V|) for every output element."""
+    ref, _ = oracle.attn_f64(Q, K, V)
+    mag = oracle.attn_absref(Q, K, V)
+    err = np.abs(got - ref)
+    worst = float((err / mag).max())
+    assert (err <= 1e-5 * mag).all(), f"{what}: worst err / magnitude = {worst:.3e}"
+    return worst
+
+
+def test_attn_workload_f32():
+    Q, K, V = inputs.attn_case_f32(1024, 64, seed=0)
+    got, st = attn_gpu_f32(Q, K, V)
+    assert st == qx.OK
+    within_tolerance(got, Q, K, V, "attn fp32 workload")
+
+
+@pytest.mark.parametrize("L,d", [(1, 64), (100, 64), (1000, 32), (129, 8), (4096, 64), (300, 48)])
+def test_attn_shapes_f32(L, d):
+    Q, K, V = inputs.attn_case_f32(L, d, seed=L + d)
+    got, st = attn_gpu_f32(Q, K, V)
+    assert st == qx.OK
+    within_tolerance(got, Q, K, V, f"attn fp32 L={L} d={d}")
+
+
+def test_attn_f32_integer_values_exact_and_deterministic():
+    # |S| <= 64*49 and 256*3136*7 < 2^24: every FP32 value on the way is an exact integer
+    Q, K, V = inputs.attn_case(256, 64, -7, 7, seed=3)
+    a, st = attn_gpu_f32(Q.float(), K.float(), V.float())
+    assert st == qx.OK
+    assert (a == oracle.attn(Q, K, V)[0]).all()
+    Qf, Kf, Vf = inputs.attn_case_f32(1024, 64, seed=8)
+    r1, _ = attn_gpu_f32(Qf, Kf, Vf)
+    r2, _ = attn_gpu_f32(Qf, Kf, Vf)
+    assert np.array_equal(r1, r2)          # fixed-order reduction of the key splits

@@ -96,3 +96,53 @@ def test_conv_range_check():
     w[3, 2, 1, 1] = -11
     _, st, _ = conv_gpu(x, w, 1, 1, (-10, 10), (-10, 10), flags=qx.FLAG_CHECK_RANGES)
     assert st == qx.ERR_CONTRACT
+
+
+# ------------------------------------------------------------ FP32 (3xTF32)
+def conv_gpu_f32(x, w, stride, pad):
+    n, c, h, wd = x.shape
+    k, _, r, s = w.shape
+    with qx.Plan(qx.conv_desc(n, c, h, wd, k, r, s, stride, pad, (0, 0), (0, 0),
+                              dtype=qx.F32)) as plan:
+        y = plan.conv2d(x.cuda(), w.cuda())
+        torch.cuda.synchronize()
+        st = plan.status()
+    return y.cpu().numpy().astype(np.float64), st
+
+
+def assert_within_tolerance(got, ref, mag, what):
+    """max |err| <= 1e-5 * sum_k |a_k||b_k| for every output element."""
+    err = np.abs(got - ref)
+    worst = float((err / np.maximum(mag, 1e-300)).max())
+    assert (err <= 1e-5 * mag).all(), f"{what}: worst err / sum|a||b| = {worst:.3e}"
+    return worst
+
+
+def test_conv_workload_f32():
+    x, w = inputs.conv_case_f32(8, 64, 56, 56, 128, 3, 3, seed=0)
+    got, st = conv_gpu_f32(x, w, 1, 1)
+    assert st == qx.OK
+    ref = oracle.conv2d_f64(x, w, 1, 1)
+    mag = oracle.conv2d_absref(x, w, 1, 1)
+    assert_within_tolerance(got, ref, mag, "conv fp32 workload")
+
+
+@pytest.mark.parametrize("shape,stride,pad", [((1, 3, 7, 9, 5, 3, 3), 1, 1),
+                                              ((3, 130, 9, 11, 200, 3, 3), 1, 1),
+                                              ((2, 16, 12, 10, 24, 1, 1), 1, 0),
+                                              ((1, 64, 30, 30, 64, 3, 3), 2, 1)])
+def test_conv_shapes_f32(shape, stride, pad):
+    n, c, h, wd, k, r, s = shape
+    x, w = inputs.conv_case_f32(n, c, h, wd, k, r, s, seed=sum(shape))
+    got, st = conv_gpu_f32(x, w, stride, pad)
+    assert st == qx.OK
+    assert_within_tolerance(got, oracle.conv2d_f64(x, w, stride, pad),
+                            oracle.conv2d_absref(x, w, stride, pad), f"conv fp32 {shape}")
+
+
+def test_conv_f32_integer_values_exact():
+    # integers of at most 11 significant bits are TF32-exact, so the result is exact
+    x, w = inputs.conv_case(2, 32, 10, 10, 16, 3, 3, -100, 100, seed=4)   # 288 * 100^2 < 2^24
+    got, st = conv_gpu_f32(x.float(), w.float(), 1, 1)
+    assert st == qx.OK
+    assert (got == oracle.conv2d(x, w, 1, 1)).all()
