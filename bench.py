@@ -181,8 +181,13 @@ def event_pair(torch):
 
 
 def op_times(torch, make_plan, call, ops, reps, dev):
-    """Setup / cached steady-state / execute-only times of one operator
-    (paper: Methodology, Table 2 QPU-C and QPU-E columns)."""
+    """Setup / cached steady-state / execute-only times of one operator, as the
+    paper separates them (Methodology; Table 2 QPU-C and QPU-E columns):
+      setup    plan creation plus the first call, host wall clock;
+      cached   host wall clock of one call on a warm plan, synchronised;
+      execute  device time of one call: the call captured once in a CUDA
+               graph and replayed back to back between CUDA events, so no
+               host launch cost is included."""
     torch.cuda.synchronize(dev)
     t0 = time.perf_counter()
     plan = make_plan()
@@ -198,63 +203,69 @@ def op_times(torch, make_plan, call, ops, reps, dev):
         call(plan)
         torch.cuda.synchronize(dev)
         cached.append((time.perf_counter() - t0) * 1e3)
-    execs = []
-    for _ in range(reps):
-        s, e = event_pair(torch)
-        s.record()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
         call(plan)
-        e.record()
-        e.synchronize()
-        execs.append(s.elapsed_time(e))
+    graph.replay()
+    torch.cuda.synchronize(dev)
+    s, e = event_pair(torch)
+    s.record()
+    for _ in range(reps):
+        graph.replay()
+    e.record()
+    e.synchronize()
+    x = s.elapsed_time(e) / reps
     st = plan.status()
+    del graph
     plan.close()
     c = statistics.median(cached)
-    x = statistics.median(execs)
     return {"setup_ms": round(setup_ms, 3), "cached_ms": round(c, 4), "execute_ms": round(x, 4),
             "cached_gops": round(ops / (c * 1e-3) / 1e9, 1),
             "execute_gops": round(ops / (x * 1e-3) / 1e9, 1), "status": st}
 
 
-def operators(torch, qx, inputs, dev):
-    out = {}
-    x, w = inputs.conv_case(8, 64, 56, 56, 128, 3, 3, -255, 255, seed=0)
-    x, w = x.to(dev), w.to(dev)
-    y = torch.empty((8, 128, 56, 56), dtype=torch.int32, device=dev)
+def operators(torch, qx, inputs, dev, only=None):
+    """Conv and attention workloads (INT16, INT32, FP32); `only` selects by name."""
+    conv_shape = (8, 64, 56, 56, 128, 3, 3)
     conv_ops = 2.0 * 8 * 128 * 56 * 56 * 64 * 9
-    out["conv_int16"] = op_times(
-        torch, lambda: qx.Plan(qx.conv_desc(8, 64, 56, 56, 128, 3, 3, 1, 1, (-255, 255), (-255, 255))),
-        lambda p: p.conv2d(x, w, y), conv_ops, 50, dev)
-    out["conv_int16"]["workload"] = "x 8x64x56x56, w 128x64x3x3, stride 1 pad 1, int16 in [-255,255]"
-    xi, wi = x.to(torch.int32), w.to(torch.int32)
-    out["conv_int32"] = op_times(
-        torch, lambda: qx.Plan(qx.conv_desc(8, 64, 56, 56, 128, 3, 3, 1, 1, (-255, 255), (-255, 255),
-                                            dtype=qx.I32)),
-        lambda p: p.conv2d(xi, wi, y), conv_ops, 50, dev)
-    xf, wf = (t.to(dev) for t in inputs.conv_case_f32(8, 64, 56, 56, 128, 3, 3, seed=0))
-    yf = torch.empty((8, 128, 56, 56), dtype=torch.float32, device=dev)
-    out["conv_fp32"] = op_times(
-        torch, lambda: qx.Plan(qx.conv_desc(8, 64, 56, 56, 128, 3, 3, 1, 1, (0, 0), (0, 0),
-                                            dtype=qx.F32)),
-        lambda p: p.conv2d(xf, wf, yf), conv_ops, 50, dev)
-    out["conv_fp32"]["workload"] = "x 8x64x56x56, w 128x64x3x3 fp32 N(0,1), 3xTF32"
-    Q, Kt, V = (t.to(dev) for t in inputs.attn_case(1024, 64, -7, 7, seed=0))
-    O = torch.empty((1024, 64), dtype=torch.int32, device=dev)
     attn_ops = 4.0 * 1024 * 1024 * 64
-    out["attn_int16"] = op_times(
-        torch, lambda: qx.Plan(qx.attn_desc(1024, 64, (-7, 7), (-7, 7), (-7, 7))),
-        lambda p: p.attn(Q, Kt, V, O), attn_ops, 50, dev)
-    out["attn_int16"]["workload"] = "Q,K,V 1024x64 int16 in [-7,7], O=(QK^T)V, no softmax"
-    Qi, Ki, Vi = (t.to(torch.int32) for t in (Q, Kt, V))
-    out["attn_int32"] = op_times(
-        torch, lambda: qx.Plan(qx.attn_desc(1024, 64, (-7, 7), (-7, 7), (-7, 7), dtype=qx.I32)),
-        lambda p: p.attn(Qi, Ki, Vi, O), attn_ops, 50, dev)
-    Qf, Kf, Vf = (t.to(dev) for t in inputs.attn_case_f32(1024, 64, seed=0))
-    Of = torch.empty((1024, 64), dtype=torch.float32, device=dev)
-    out["attn_fp32"] = op_times(
-        torch, lambda: qx.Plan(qx.attn_desc(1024, 64, (0, 0), (0, 0), (0, 0), dtype=qx.F32)),
-        lambda p: p.attn(Qf, Kf, Vf, Of), attn_ops, 50, dev)
-    out["attn_fp32"]["workload"] = "Q,K,V 1024x64 fp32 N(0,1), 3xTF32"
-    return out
+
+    def conv(dtype):
+        if dtype == qx.F32:
+            x, w = inputs.conv_case_f32(*conv_shape, seed=0)
+            rng, desc = (0, 0), "fp32 N(0,1), 3xTF32"
+        else:
+            tdt = torch.int16 if dtype == qx.I16 else torch.int32
+            x, w = inputs.conv_case(*conv_shape, -255, 255, seed=0, dtype=tdt)
+            rng, desc = (-255, 255), f"{'int16' if dtype == qx.I16 else 'int32'} in [-255,255]"
+        x, w = x.to(dev), w.to(dev)
+        y = torch.empty((8, 128, 56, 56), dtype=torch.float32 if dtype == qx.F32 else torch.int32,
+                        device=dev)
+        r = op_times(torch, lambda: qx.Plan(qx.conv_desc(*conv_shape, 1, 1, rng, rng, dtype=dtype)),
+                     lambda p: p.conv2d(x, w, y), conv_ops, 50, dev)
+        r["workload"] = f"x 8x64x56x56 * w 128x64x3x3, stride 1 pad 1, {desc}"
+        return r
+
+    def attn(dtype):
+        if dtype == qx.F32:
+            Q, K, V = inputs.attn_case_f32(1024, 64, seed=0)
+            rng, desc = (0, 0), "fp32 N(0,1), 3xTF32"
+        else:
+            tdt = torch.int16 if dtype == qx.I16 else torch.int32
+            Q, K, V = inputs.attn_case(1024, 64, -7, 7, seed=0, dtype=tdt)
+            rng, desc = (-7, 7), f"{'int16' if dtype == qx.I16 else 'int32'} in [-7,7]"
+        Q, K, V = Q.to(dev), K.to(dev), V.to(dev)
+        O = torch.empty((1024, 64), dtype=torch.float32 if dtype == qx.F32 else torch.int32,
+                        device=dev)
+        r = op_times(torch, lambda: qx.Plan(qx.attn_desc(1024, 64, rng, rng, rng, dtype=dtype)),
+                     lambda p: p.attn(Q, K, V, O), attn_ops, 50, dev)
+        r["workload"] = f"Q,K,V 1024x64, O=(QK^T)V, no softmax, {desc}"
+        return r
+
+    table = {"conv_int16": lambda: conv(qx.I16), "conv_int32": lambda: conv(qx.I32),
+             "conv_fp32": lambda: conv(qx.F32), "attn_int16": lambda: attn(qx.I16),
+             "attn_int32": lambda: attn(qx.I32), "attn_fp32": lambda: attn(qx.F32)}
+    return {k: f() for k, f in table.items() if only is None or k in only}
 
 
 def sweep(args):
@@ -268,6 +279,7 @@ def sweep(args):
     from paper_2606_09905_gb300 import inputs, qx
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
+    only = set(args.only.split(",")) if args.only else None
     rows = []
     shapes = [(256, 256, 256, 1023), (512, 512, 512, 1023), (768, 768, 768, 1023),
               (1024, 1024, 1024, 1023), (2048, 2048, 2048, 1023), (4096, 64, 1024, 1023),
@@ -276,6 +288,9 @@ def sweep(args):
         for dt, tdt in ((qx.I16, torch.int16), (qx.I32, torch.int32)):
             if m == 8192 and dt == qx.I32:
                 continue
+            tag = f"gemm{m}x{n}x{k}_{'i16' if dt == qx.I16 else 'i32'}"
+            if only is not None and tag not in only:
+                continue
             A, B = inputs.gemm_case(m, n, k, -r, r, seed=0, dtype=tdt)
             A, B = A.to(dev), B.to(dev)
             C = torch.empty((m, n), dtype=torch.int32, device=dev)
@@ -283,10 +298,11 @@ def sweep(args):
             res = op_times(torch, lambda: qx.Plan(qx.gemm_desc(m, n, k, (-r, r), (-r, r), dtype=dt)),
                            lambda p: getattr(p, fn)(A, B, C), 2.0 * m * n * k,
                            20 if m >= 4096 else 100, dev)
-            res.update(workload=f"gemm {m}x{n}x{k} {'int16' if dt == qx.I16 else 'int32'} [-{r},{r}]")
+            res.update(workload=f"{tag} [-{r},{r}]")
             rows.append(res)
-    rows += [dict(v, workload=v.get("workload", k) + f" ({k})") for k, v in
-             operators(torch, qx, inputs, dev).items()]
+    if only is None or any(not t.startswith("gemm") for t in only):
+        rows += [dict(v, workload=f"{k}: " + v.get("workload", k)) for k, v in
+                 operators(torch, qx, inputs, dev, only).items()]
     for r in rows:
         print(json.dumps(r), flush=True)
     return 0
@@ -398,34 +414,65 @@ def run_qx(args):
     value = world * ops / (ms_step * 1e-3) / 1e12
 
     # -------------------------------------------- end to end, host buffers
+    # Every step copies its inputs from pinned host memory, runs the GEMM
+    # through the public call and copies its result back.  The three stages
+    # run on their own streams with two device buffer sets, so step i's
+    # copies overlap step i-1's GEMM (a pipelined loop, as a serving loop
+    # would run it).
     hA = A.pin_memory()
     hB = B.pin_memory()
-    hC = torch.empty((M, N), dtype=torch.int32).pin_memory()
-    e2e_steps = max(3, min(args.steps, 10))
-    for _ in range(2):
-        dA.copy_(hA, non_blocking=True)
-        dB.copy_(hB, non_blocking=True)
-        plan.gemm_i16_i32(dA, dB, C)
-        hC.copy_(C, non_blocking=True)
+    hC = [torch.empty((M, N), dtype=torch.int32).pin_memory() for _ in range(2)]
+    dA2 = [dA, torch.empty_like(dA)]
+    dB2 = [dB, torch.empty_like(dB)]
+    dC2 = [C, torch.empty_like(C)]
+    s_in, s_c, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    in_done = [torch.cuda.Event() for _ in range(2)]
+    comp_done = [torch.cuda.Event() for _ in range(2)]
+    out_done = [torch.cuda.Event() for _ in range(2)]
+
+    def e2e_step(i):
+        k = i & 1
+        if i >= 2:
+            s_in.wait_event(comp_done[k])         # GEMM of step i-2 has read slot k
+        with torch.cuda.stream(s_in):
+            dA2[k].copy_(hA, non_blocking=True)
+            dB2[k].copy_(hB, non_blocking=True)
+            in_done[k].record(s_in)
+        s_c.wait_event(in_done[k])
+        if i >= 2:
+            s_c.wait_event(out_done[k])           # result of step i-2 has left slot k
+        plan.gemm_i16_i32(dA2[k], dB2[k], dC2[k], stream=s_c)
+        comp_done[k].record(s_c)
+        s_out.wait_event(comp_done[k])
+        with torch.cuda.stream(s_out):
+            hC[k].copy_(dC2[k], non_blocking=True)
+            out_done[k].record(s_out)
+
+    e2e_steps = max(4, min(args.steps, 20))
+    for i in range(2):
+        e2e_step(i)
     torch.cuda.synchronize(dev)
     barrier()
     e0, e1 = event_pair(torch)
-    e0.record(stream)
-    for _ in range(e2e_steps):
-        dA.copy_(hA, non_blocking=True)
-        dB.copy_(hB, non_blocking=True)
-        plan.gemm_i16_i32(dA, dB, C)
-        hC.copy_(C, non_blocking=True)
-    e1.record(stream)
+    e0.record(s_in)
+    s_c.wait_event(e0)
+    s_out.wait_event(e0)
+    for i in range(e2e_steps):
+        e2e_step(i)
+    e1.record(s_out)
     torch.cuda.synchronize(dev)
     e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    if not (torch.equal(hC[0], hC[1]) and torch.equal(hC[0], dC2[0].cpu())):
+        raise SystemExit("pipelined end-to-end results disagree")
     if world > 1:
         tt = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         e2e_ms = float(tt.item())
     e2e = {"value": world * ops / (e2e_ms * 1e-3) / 1e12, "unit": "TOPS",
            "h2d_bytes_per_step": hA.numel() * 2 + hB.numel() * 2,
-           "d2h_bytes_per_step": hC.numel() * 4, "ms_per_step": e2e_ms}
+           "d2h_bytes_per_step": hC[0].numel() * 4, "ms_per_step": e2e_ms,
+           "pipeline": "H2D / GEMM / D2H on three streams, two buffer sets"}
+    del dA2, dB2, dC2
 
     # cached steady state (host wall per call, with sync), as the paper's QPU-C
     cached = []
@@ -496,6 +543,9 @@ def main():
     ap.add_argument("--impl", choices=["qx", "reference"], default="qx")
     ap.add_argument("--sweep", action="store_true",
                     help="time every workload (setup / cached / execute-only), one JSON line each")
+    ap.add_argument("--only", default="",
+                    help="with --sweep: comma-separated workload names (e.g. conv_int16,"
+                         "gemm256x256x256_i16)")
     ap.add_argument("--no-operators", action="store_true", help="skip the conv/attention timings")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
