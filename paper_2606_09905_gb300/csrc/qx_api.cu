@@ -40,8 +40,8 @@ cudaError_t attn_prepare();
 cudaError_t attn_f32_prepare();
 cudaError_t attn_f32_launch(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_pack_attn_f32(const float *Q, const float *K, const float *V, int L, int d, int Lp,
-                                 float *q, float *k, float *vt, unsigned *counters, int q_tiles,
-                                 int num_sms, cudaStream_t st);
+                                 float *q, float *k, float *vt, int num_sms, cudaStream_t st);
+int attn_max_cluster();
 cudaError_t attn_launch(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_pack_gemm(bool i32, const void *A, const void *B, int64_t lda, int64_t ldb,
                              int M, int N, int K, int Kp, __half *a_planes, __half *bt_planes,
@@ -513,6 +513,22 @@ static qx_status build_conv(qx_plan p) {
     return QX_OK;
 }
 
+// Key splits of one query tile form one cluster (at most attn_max_cluster()
+// CTAs); each CTA takes a run of whole key blocks.
+static void attn_splits(int key_blocks, int q_tiles, int num_sms, int max_blocks_per_cta, int *splits,
+                        int *per) {
+    int cs = std::max(1, std::min({attn_max_cluster(), key_blocks,
+                                   std::max(1, num_sms / std::max(1, q_tiles))}));
+    int blocks = (key_blocks + cs - 1) / cs;
+    if (blocks > max_blocks_per_cta) {
+        cs = std::min(attn_max_cluster(), (key_blocks + max_blocks_per_cta - 1) / max_blocks_per_cta);
+        blocks = (key_blocks + cs - 1) / cs;
+    }
+    cs = (key_blocks + blocks - 1) / blocks;   // no CTA without keys
+    *splits = cs;
+    *per = blocks;
+}
+
 static qx_status build_attn_f32(qx_plan p) {
     const qx_plan_desc &d = p->desc;
     p->dp = 64;
@@ -522,18 +538,13 @@ static qx_status build_attn_f32(qx_plan p) {
     a.L = int(d.L);
     a.d = int(d.d);
     a.q_tiles = int((d.L + 127) / 128);
-    const int key_blocks = int((d.L + 31) / 32);
-    int splits = std::max(1, std::min(key_blocks, (p->num_sms + a.q_tiles - 1) / a.q_tiles));
-    const int per = (key_blocks + splits - 1) / splits;
-    splits = (key_blocks + per - 1) / per;
+    int splits = 1, per = 1;
+    attn_splits(int((d.L + 31) / 32), a.q_tiles, p->num_sms, INT32_MAX, &splits, &per);
     a.key_splits = splits;
     a.keys_per_split = per * 32;
     const size_t qk_bytes = size_t(2) * d.L * 64 * 4;
     const size_t vt_bytes = size_t(2) * 64 * p->Lp * 4;
-    const size_t part_bytes = size_t(a.q_tiles) * splits * 128 * 64 * 4;
-    const size_t cnt_bytes = size_t(a.q_tiles) * 4;
-    p->ws_bytes = 256 + 2 * align256(qk_bytes) + align256(vt_bytes) + align256(part_bytes) +
-                  align256(cnt_bytes);
+    p->ws_bytes = 256 + 2 * align256(qk_bytes) + align256(vt_bytes);
     QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
     char *base = static_cast<char *>(p->ws);
     p->err = reinterpret_cast<int *>(base);
@@ -543,10 +554,6 @@ static qx_status build_attn_f32(qx_plan p) {
     p->fk = reinterpret_cast<float *>(base + off);
     off += align256(qk_bytes);
     p->fvt = reinterpret_cast<float *>(base + off);
-    off += align256(vt_bytes);
-    a.partial = reinterpret_cast<float *>(base + off);
-    off += align256(part_bytes);
-    a.counters = reinterpret_cast<unsigned *>(base + off);
     QX_CUDA(cudaMemset(p->ws, 0, p->ws_bytes), "workspace reset");
     {
         const uint64_t dims[3] = {64, uint64_t(d.L), 2};
@@ -611,13 +618,12 @@ static qx_status build_attn(qx_plan p) {
     a.q_tiles = int((d.L + 127) / 128);
     const int key_blocks = int((d.L + 63) / 64);
     const int max_blocks = std::max(1, p->max_keys / 64);
-    int splits = std::max(1, std::min(key_blocks, (p->num_sms + a.q_tiles - 1) / a.q_tiles));
-    int per = (key_blocks + splits - 1) / splits;
-    if (per > max_blocks) {
-        per = max_blocks;
-        splits = (key_blocks + per - 1) / per;
-    }
-    splits = (key_blocks + per - 1) / per;
+    int splits = 1, per = 1;
+    attn_splits(key_blocks, a.q_tiles, p->num_sms, max_blocks, &splits, &per);
+    if (per > max_blocks)
+        return fail(QX_ERR_UNSUPPORTED,
+                    "L = %lld needs more than %d exact key chunks per query tile",
+                    (long long)d.L, attn_max_cluster());
     a.key_splits = splits;
     a.keys_per_split = per * 64;
     a.s_shift = p->s_shift;
@@ -793,8 +799,7 @@ static qx_status pack(qx_plan p, const void *a, const void *b, const void *c, cu
                 QX_CUDA(launch_pack_attn_f32(static_cast<const float *>(a),
                                              static_cast<const float *>(b),
                                              static_cast<const float *>(c), int(d.L), int(d.d),
-                                             p->Lp, p->fq, p->fk, p->fvt, p->attn.counters,
-                                             p->attn.q_tiles, p->num_sms, st),
+                                             p->Lp, p->fq, p->fk, p->fvt, p->num_sms, st),
                         "operand packing launch");
                 return QX_OK;
             }
@@ -844,7 +849,6 @@ static qx_status run_packed(qx_plan p, void *out, cudaStream_t st) {
                 QX_CUDA(attn_f32_launch(a, st), "attention launch");
                 return QX_OK;
             }
-            QX_CUDA(cudaMemsetAsync(out, 0, size_t(d.L) * d.d * 4, st), "zero output");
             QX_CUDA(attn_launch(a, st), "attention launch");
             return QX_OK;
         }

@@ -71,16 +71,12 @@ struct AttnArgs {
     CUtensorMap tm_q;         // Q   (L x d): fp16 2-D, or fp32 3-D (d, L, big/small)
     CUtensorMap tm_k;         // K   (L x d): same
     CUtensorMap tm_vt;        // V^T (d x L): fp16 2-D, or fp32 3-D (L, d, big/small)
-    void *out;                // O (L x d): int32 (zeroed before the launch) or float
+    void *out;                // O (L x d): int32 or float
     int *err;
     int L, d;
-    int q_tiles, key_splits, keys_per_split;
+    int q_tiles, key_splits, keys_per_split;   // key_splits = cluster size (<= 8)
     int s_shift;              // digit width of the S limbs (integer kind)
     int o_chunk_kb;           // key-blocks per FP32 chunk of the second product
-    // FP32 kind: per-CTA partial O (q_tiles x key_splits x 128 x 64 floats) and
-    // one arrival counter per query tile (zero between calls)
-    float *partial;
-    unsigned *counters;
 };
 
 }  // namespace qx

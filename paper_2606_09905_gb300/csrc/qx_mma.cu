@@ -125,6 +125,8 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    // the packed operands come from the kernel launched just before this one
+    pdl_wait();
 
     if (warp == 0) {
         if (lane == 0) {
@@ -358,8 +360,7 @@ static cudaError_t prepare_t() {
 template <int NA, int NB, int KIND = kKindExact>
 static cudaError_t launch_t(const MmaArgs &a, int grid, cudaStream_t stream) {
     using T = TileCfg<NA, NB, KIND>;
-    limb_gemm_kernel<NA, NB, KIND><<<grid, T::THREADS, T::SMEM, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(limb_gemm_kernel<NA, NB, KIND>, grid, T::THREADS, T::SMEM, stream, a);
 }
 
 #define QX_LIMB_DISPATCH(FN, ...)                                          \

@@ -82,6 +82,7 @@ struct GemmPackArgs {
 
 template <typename T, int NA, int NB>
 __global__ void __launch_bounds__(256) pack_gemm_kernel(const GemmPackArgs p) {
+    pdl_launch_dependents();
     __shared__ int32_t tile[64][65];
     const T *A = static_cast<const T *>(p.A);
     const T *B = static_cast<const T *>(p.B);
@@ -145,6 +146,7 @@ struct ConvPackArgs {
 
 template <typename T, int NX, int NW>
 __global__ void __launch_bounds__(256) pack_conv_kernel(const ConvPackArgs p) {
+    pdl_launch_dependents();
     __shared__ int32_t tile[64][65];
     const T *X = static_cast<const T *>(p.x);
     const T *W = static_cast<const T *>(p.w);
@@ -228,6 +230,7 @@ __device__ __forceinline__ void store_split8(float *plane0, int64_t plane_stride
 }
 
 __global__ void __launch_bounds__(256) pack_conv_f32_kernel(const ConvPackF32Args p) {
+    pdl_launch_dependents();
     __shared__ float tile[64][65];
     const int HW = p.h * p.wd;
     if (int(blockIdx.x) < p.x_blocks) {
@@ -289,6 +292,7 @@ struct AttnPackArgs {
 
 template <typename T>
 __global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
+    pdl_launch_dependents();
     __shared__ int32_t tile[64][65];
     const T *Q = static_cast<const T *>(p.Q);
     const T *K = static_cast<const T *>(p.K);
@@ -343,22 +347,18 @@ __global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
 
 // ------------------------------------------------ attention, FP32 kind
 // Q, K (L x d) -> big/small TF32 planes [2][L][64] (zero columns beyond d);
-// V -> V^T planes [2][64][Lp]; the per-query-tile arrival counters of the
-// attention kernel are zeroed here, before every launch.
+// V -> V^T planes [2][64][Lp].
 struct AttnPackF32Args {
     const float *Q, *K, *V;
     int L, d, Lp;
     float *q, *k, *vt;
-    unsigned *counters;
-    int q_tiles;
     int qk_blocks, v_tiles_l;
 };
 
 __global__ void __launch_bounds__(256) pack_attn_f32_kernel(const AttnPackF32Args p) {
+    pdl_launch_dependents();
     __shared__ float tile[64][65];
     if (int(blockIdx.x) < p.qk_blocks) {
-        if (blockIdx.x == 0)
-            for (int i = threadIdx.x; i < p.q_tiles; i += blockDim.x) p.counters[i] = 0u;
         const int64_t items = int64_t(2) * p.L * 8;            // 8 groups of 8 columns
         for (int64_t it = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; it < items;
              it += int64_t(p.qk_blocks) * blockDim.x) {
@@ -546,8 +546,7 @@ cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void 
 
 namespace qx {
 cudaError_t launch_pack_attn_f32(const float *Q, const float *K, const float *V, int L, int d, int Lp,
-                                 float *q, float *k, float *vt, unsigned *counters, int q_tiles,
-                                 int num_sms, cudaStream_t st) {
+                                 float *q, float *k, float *vt, int num_sms, cudaStream_t st) {
     AttnPackF32Args p;
     p.Q = Q;
     p.K = K;
@@ -558,8 +557,6 @@ cudaError_t launch_pack_attn_f32(const float *Q, const float *K, const float *V,
     p.q = q;
     p.k = k;
     p.vt = vt;
-    p.counters = counters;
-    p.q_tiles = q_tiles;
     const int64_t items = int64_t(2) * L * 8;
     int64_t blocks = (items + 255) / 256;
     if (blocks > num_sms) blocks = num_sms;
