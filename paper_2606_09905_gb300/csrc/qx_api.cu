@@ -11,6 +11,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -311,6 +312,17 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
 
 static size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
 
+// Width (in N-side tiles) of the tile groups the persistent kernel walks.  The
+// CTAs resident at one time cover about G N-side tiles x grid/G M-side tiles,
+// so each wave reads G N-side panels and grid/G M-side panels (all of K);
+// G = sqrt(grid * M-panel bytes / N-panel bytes) minimises that traffic.
+static int tile_group(int grid, int tiles_n, int nb, int na, int mr) {
+    const double m_panel = double(kBM) * nb;     // bytes per K of one M-side tile
+    const double n_panel = double(mr) * na;      // bytes per K of one N-side tile
+    int g = int(std::sqrt(double(grid) * m_panel / n_panel));
+    return std::max(1, std::min(g, tiles_n));
+}
+
 // ----------------------------------------------------------- device scope
 struct DeviceScope {
     int prev = -1;
@@ -371,11 +383,11 @@ static qx_status build_gemm(qx_plan p) {
     a.chunk_kb = int(s.chunk_kb);
     a.tiles_m = int((d.N + kBM - 1) / kBM);
     a.tiles_n = int((d.M + mr - 1) / mr);
-    a.group_n = std::max(1, std::min(16, a.tiles_n));
     a.shift_n = s.n.shift;
     a.shift_m = s.m.shift;
     const int tiles = a.tiles_m * a.tiles_n;
     p->grid = std::max(1, std::min(tiles, p->num_sms));
+    a.group_n = tile_group(p->grid, a.tiles_n, nb, na, mr);
     QX_CUDA(limb_gemm_prepare(na, nb), "kernel attributes");
     return QX_OK;
 }

@@ -78,6 +78,7 @@ struct GemmPackArgs {
     int a_blocks;          // blocks [0, a_blocks) pack A, the rest transpose B
     int b_tiles_n;         // B tiles along N (64 wide)
     int vec_a;             // A rows 16-byte aligned for 8-element loads
+    int vec_b;             // B rows likewise
 };
 
 template <typename T, int NA, int NB>
@@ -105,18 +106,27 @@ __global__ void __launch_bounds__(256) pack_gemm_kernel(const GemmPackArgs p) {
         }
         return;
     }
-    // B (K x N, row-major) -> NB planes of N x Kp: 64 x 64 tiles through smem
+    // B (K x N, row-major) -> NB planes of N x Kp: 64 x 64 tiles through smem,
+    // read 8 consecutive n per thread (16-byte loads where B allows them)
     const int t = int(blockIdx.x) - p.a_blocks;
     const int n0 = (t % p.b_tiles_n) * 64;
     const int k0 = (t / p.b_tiles_n) * 64;
-    for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
-        const int kr = i >> 6, nc = i & 63;
-        int32_t v = 0;
-        if (k0 + kr < p.K && n0 + nc < p.N) {
-            v = int32_t(B[int64_t(k0 + kr) * p.ldb + n0 + nc]);
-            p.cb.test(v, p.err);
+    for (int i = threadIdx.x; i < 64 * 8; i += blockDim.x) {
+        const int kr = i >> 3, ng = i & 7;
+        const int k = k0 + kr, n = n0 + ng * 8;
+        int32_t v[8];
+        if (k < p.K && n < p.N) {
+            const int valid = min(8, p.N - n);
+            load8<T>(B + int64_t(k) * p.ldb + n, p.vec_b && valid == 8, valid, v);
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                if (e < valid) p.cb.test(v[e], p.err);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = 0;
         }
-        tile[kr][nc] = v;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) tile[kr][ng * 8 + e] = v[e];
     }
     __syncthreads();
     const int64_t plane_stride = int64_t(p.N) * p.Kp;
@@ -429,6 +439,7 @@ cudaError_t launch_pack_gemm(bool i32, const void *A, const void *B, int64_t lda
     p.err = err;
     const int esz = i32 ? 4 : 2;
     p.vec_a = (reinterpret_cast<uintptr_t>(A) % 16 == 0) && ((lda * esz) % 16 == 0);
+    p.vec_b = (reinterpret_cast<uintptr_t>(B) % 16 == 0) && ((ldb * esz) % 16 == 0);
     const int64_t a_items = int64_t(M) * ((K + 7) / 8);
     const int64_t a_blocks = (a_items + 255) / 256;
     p.a_blocks = int(a_blocks < int64_t(num_sms) * 8 ? a_blocks : int64_t(num_sms) * 8);
