@@ -224,8 +224,23 @@ def op_times(torch, make_plan, call, ops, reps, dev):
             "execute_gops": round(ops / (x * 1e-3) / 1e9, 1), "status": st}
 
 
+def op_roofline(flops_tensor: float, tensor_peak_tflops: float, hbm_bytes: float,
+                hbm_gbs: float, exec_ms: float) -> dict:
+    """Roofline of one operator call: the slower of its tensor work (FLOPs of
+    the exact scheme's MMAs at the peak of their kind) and its algorithmic
+    bytes (operands read once, output written once) at HBM bandwidth."""
+    t_tensor = flops_tensor / (tensor_peak_tflops * 1e12) * 1e3
+    t_hbm = hbm_bytes / (hbm_gbs * 1e9) * 1e3
+    bound = "tensor" if t_tensor >= t_hbm else "hbm"
+    t_roof = max(t_tensor, t_hbm)
+    return {"bound": bound, "roof_us": round(t_roof * 1e3, 3),
+            "frac": round(t_roof / exec_ms, 4) if exec_ms > 0 else None,
+            "tensor_us": round(t_tensor * 1e3, 3), "hbm_us": round(t_hbm * 1e3, 3)}
+
+
 def operators(torch, qx, inputs, dev, only=None):
     """Conv and attention workloads (INT16, INT32, FP32); `only` selects by name."""
+    peaks = load_peaks()
     conv_shape = (8, 64, 56, 56, 128, 3, 3)
     conv_ops = 2.0 * 8 * 128 * 56 * 56 * 64 * 9
     attn_ops = 4.0 * 1024 * 1024 * 64
@@ -241,9 +256,14 @@ def operators(torch, qx, inputs, dev, only=None):
         x, w = x.to(dev), w.to(dev)
         y = torch.empty((8, 128, 56, 56), dtype=torch.float32 if dtype == qx.F32 else torch.int32,
                         device=dev)
-        r = op_times(torch, lambda: qx.Plan(qx.conv_desc(*conv_shape, 1, 1, rng, rng, dtype=dtype)),
-                     lambda p: p.conv2d(x, w, y), conv_ops, 50, dev)
+        plan_desc = qx.conv_desc(*conv_shape, 1, 1, rng, rng, dtype=dtype)
+        r = op_times(torch, lambda: qx.Plan(plan_desc), lambda p: p.conv2d(x, w, y), conv_ops, 50, dev)
         r["workload"] = f"x 8x64x56x56 * w 128x64x3x3, stride 1 pad 1, {desc}"
+        m = qx.query(plan_desc)[0]["mma_per_kstep"]
+        esz = x.element_size()
+        nbytes = x.numel() * esz + w.numel() * esz + y.numel() * 4
+        tensor_peak = peaks["bf16_tflops"] / (2.0 if dtype == qx.F32 else 1.0)   # TF32 runs at half rate
+        r["roofline"] = op_roofline(m * conv_ops, tensor_peak, nbytes, peaks["hbm_gbs"], r["execute_ms"])
         return r
 
     def attn(dtype):
@@ -257,9 +277,15 @@ def operators(torch, qx, inputs, dev, only=None):
         Q, K, V = Q.to(dev), K.to(dev), V.to(dev)
         O = torch.empty((1024, 64), dtype=torch.float32 if dtype == qx.F32 else torch.int32,
                         device=dev)
-        r = op_times(torch, lambda: qx.Plan(qx.attn_desc(1024, 64, rng, rng, rng, dtype=dtype)),
-                     lambda p: p.attn(Q, K, V, O), attn_ops, 50, dev)
+        plan_desc = qx.attn_desc(1024, 64, rng, rng, rng, dtype=dtype)
+        r = op_times(torch, lambda: qx.Plan(plan_desc), lambda p: p.attn(Q, K, V, O), attn_ops, 50, dev)
         r["workload"] = f"Q,K,V 1024x64, O=(QK^T)V, no softmax, {desc}"
+        s0, s1 = qx.query(plan_desc)
+        flops = (s0["mma_per_kstep"] + s1["mma_per_kstep"]) * attn_ops / 2.0
+        esz = Q.element_size()
+        nbytes = 3 * Q.numel() * esz + O.numel() * 4
+        tensor_peak = peaks["bf16_tflops"] / (2.0 if dtype == qx.F32 else 1.0)
+        r["roofline"] = op_roofline(flops, tensor_peak, nbytes, peaks["hbm_gbs"], r["execute_ms"])
         return r
 
     table = {"conv_int16": lambda: conv(qx.I16), "conv_int32": lambda: conv(qx.I32),
@@ -280,6 +306,7 @@ def sweep(args):
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     only = set(args.only.split(",")) if args.only else None
+    peaks = load_peaks()
     rows = []
     shapes = [(256, 256, 256, 1023), (512, 512, 512, 1023), (768, 768, 768, 1023),
               (1024, 1024, 1024, 1023), (2048, 2048, 2048, 1023), (4096, 64, 1024, 1023),
@@ -299,6 +326,11 @@ def sweep(args):
                            lambda p: getattr(p, fn)(A, B, C), 2.0 * m * n * k,
                            20 if m >= 4096 else 100, dev)
             res.update(workload=f"{tag} [-{r},{r}]")
+            mlimb = qx.query(qx.gemm_desc(m, n, k, (-r, r), (-r, r), dtype=dt))[0]["mma_per_kstep"]
+            esz = 2 if dt == qx.I16 else 4
+            res["roofline"] = op_roofline(mlimb * 2.0 * m * n * k, peaks["bf16_tflops"],
+                                          (m * k + k * n) * esz + m * n * 4, peaks["hbm_gbs"],
+                                          res["execute_ms"])
             rows.append(res)
     if only is None or any(not t.startswith("gemm") for t in only):
         rows += [dict(v, workload=f"{k}: " + v.get("workload", k)) for k, v in

@@ -5,7 +5,7 @@
 #include <cuda_runtime.h>
 #include <cstdint>
 
-#include "../../include/qx.h"
+#include "qx.h"  // include/ is on the include path
 
 namespace qx {
 

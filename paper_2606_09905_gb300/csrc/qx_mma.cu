@@ -105,6 +105,11 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
     const int ntiles = a.tiles_m * a.tiles_n;
 
     if (threadIdx.x == 0) {
+        // descriptor fetches overlap the prologue (the maps are launch
+        // parameters, not data of the previous kernel)
+        tma_prefetch(&a.tm_m[0]);
+        if (NB > 1) tma_prefetch(&a.tm_m[1]);
+        tma_prefetch(&a.tm_n);
         for (int s = 0; s < T::STAGES; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
@@ -131,9 +136,6 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
     if (warp == 0) {
         if (lane == 0) {
             // ------------------------------------------------ TMA producer
-            tma_prefetch(&a.tm_m[0]);
-            if (NB > 1) tma_prefetch(&a.tm_m[1]);
-            tma_prefetch(&a.tm_n);
             int stage = 0;
             uint32_t phase = 0;
             long long issued = 0;

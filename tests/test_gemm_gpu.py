@@ -190,3 +190,22 @@ def test_gemm_8192_sampled_rows_and_freivalds():
     for _ in range(4):
         x = rng.choice([-1, 1], size=(N, 2)).astype(np.int64)
         assert (a @ (b @ x) == got @ x).all()
+
+
+def test_full_smul24_operand_range_int32():
+    """INT32 operands over the whole 24-bit signed range of the smul24 contract
+    (|a|, |b| < 2^23): four digits of A times two of B; the product is exact
+    modulo 2^32 (it leaves int32, so the oracle's value is reduced the same way)."""
+    r = (-(2**23 - 1), 2**23 - 1)
+    info = qx.query(qx.gemm_desc(130, 140, 300, r, r, dtype=qx.I32))[0]
+    assert (info["limbs_a"], info["limbs_b"]) == (4, 2)
+    g = torch.Generator().manual_seed(23)
+    A = torch.randint(r[0], r[1] + 1, (130, 300), generator=g, dtype=torch.int32)
+    B = torch.randint(r[0], r[1] + 1, (300, 140), generator=g, dtype=torch.int32)
+    A[0, :] = r[1]
+    A[1, :] = r[0]
+    B[:, 0] = r[1]
+    ref, _ = oracle.gemm(A, B)
+    got, st, _ = gemm_gpu(A, B, r, r, dtype=qx.I32)
+    assert st == qx.OK
+    assert_exact(got, wrap32(ref), "smul24 range")
