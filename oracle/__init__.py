@@ -16,6 +16,9 @@ Definitions (paper: Abstract, Methodology paragraph, Table 1, Table 2):
   accumulation contract of the Methodology paragraph).
 * ``conv2d``  direct NCHW/KCRS cross-correlation with zero padding, no bias.
 * ``attn``    S = Q K^T then O = S V, no softmax and no scale.
+* ``minmax``  smallest and largest element (Table 2 min/max rows).
+* ``pool2d``  NCHW max / average pooling without padding (Table 2 pooling
+  rows); integer averages are floor(window sum / window size).
 * ``*_f64``   the same three definitions in float64; ``*_absref`` applies them
   to element-wise absolute values, giving the per-element magnitude
   sum |a_k||b_k| that the FP32 tolerance is stated against.
@@ -65,6 +68,10 @@ def _load():
             lib.qxo_gemm_f64.argtypes = [_i64, _i64, _i64, _p, _i64, _p, _i64, _p, _i64]
             lib.qxo_conv2d_f64.argtypes = [_i64] * 9 + [_p, _p, _p]
             lib.qxo_attn_f64.argtypes = [_i64, _i64, _p, _p, _p, _p, _p]
+            lib.qxo_minmax_i64.argtypes = [_i64, _p, _p, _p]
+            lib.qxo_minmax_f64.argtypes = [_i64, _p, _p, _p]
+            lib.qxo_pool2d_i64.argtypes = [_i64] * 7 + [ctypes.c_int, _p, _p]
+            lib.qxo_pool2d_f64.argtypes = [_i64] * 7 + [ctypes.c_int, _p, _p]
             _lib = lib
     return _lib
 
@@ -211,3 +218,42 @@ def attn_absref(Q, K, V):
     measured against (it carries the first product's error into the second)."""
     O, _ = attn_f64(np.abs(_as_f64(Q)), np.abs(_as_f64(K)), np.abs(_as_f64(V)))
     return O
+
+
+# ------------------------------------------------ memory-bound operators
+def minmax(x):
+    """(min, max) of all elements: exact for integers, float64 for floats."""
+    a = _np(x).reshape(-1)
+    if a.size == 0:
+        raise ValueError("empty input")
+    if a.dtype.kind in "iu":
+        a = _as_i32(a)
+        lo, hi = ctypes.c_int64(0), ctypes.c_int64(0)
+        _load().qxo_minmax_i64(a.size, _ptr(a), ctypes.byref(lo), ctypes.byref(hi))
+        return int(lo.value), int(hi.value)
+    a = _as_f64(a)
+    lo, hi = ctypes.c_double(0), ctypes.c_double(0)
+    _load().qxo_minmax_f64(a.size, _ptr(a), ctypes.byref(lo), ctypes.byref(hi))
+    return float(lo.value), float(hi.value)
+
+
+def pool2d(x, kh: int = 2, kw: int = 2, stride: int = 2, mode: str = "max"):
+    """NCHW pooling, no padding.  Integers: int64 result (average = floor);
+    floats: float64 result."""
+    a = _np(x)
+    if a.ndim != 4 or kh < 1 or kw < 1 or stride < 1 or mode not in ("max", "avg"):
+        raise ValueError("bad pooling arguments")
+    n, c, h, w = a.shape
+    if h < kh or w < kw:
+        raise ValueError("window larger than the image")
+    P, Q = (h - kh) // stride + 1, (w - kw) // stride + 1
+    is_max = 1 if mode == "max" else 0
+    if a.dtype.kind in "iu":
+        a = _as_i32(a)
+        y = np.zeros((n, c, P, Q), dtype=np.int64)
+        _load().qxo_pool2d_i64(n, c, h, w, kh, kw, stride, is_max, _ptr(a), _ptr(y))
+    else:
+        a = _as_f64(a)
+        y = np.zeros((n, c, P, Q), dtype=np.float64)
+        _load().qxo_pool2d_f64(n, c, h, w, kh, kw, stride, is_max, _ptr(a), _ptr(y))
+    return y

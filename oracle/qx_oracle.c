@@ -26,6 +26,8 @@
  *     (Methodology; Table 2), computed as written: first S = Q K^T, then
  *     O = S V.
  *   - FP64 versions of the three operators for the FP32 variants of Table 2.
+ *   - The memory-bound operators of Table 2: min/max reduction and 2-D max /
+ *     average pooling (end of the file).
  *     The tolerance reference sum_k |a_k||b_k| is the same routine applied to
  *     element-wise absolute values (the Python wrapper does that).
  *
@@ -202,4 +204,82 @@ void qxo_attn_f64(int64_t L, int64_t d,
             O[i * d + cc] = acc;
         }
     if (!S) free(Sb);
+}
+
+/* ---- memory-bound operators of Table 2 (min/max reduction, pooling) ----
+ * Min/max: the smallest and the largest element of x[0..n).
+ * Pooling: NCHW input, kernel kh x kw, stride st, no padding, output
+ * P = (h - kh) / st + 1 rows, Q likewise.  Max pooling takes the window
+ * maximum; average pooling of integers takes floor(window sum / (kh*kw))
+ * (the reading for the paper's INT32 AvgPool, equal to an arithmetic right
+ * shift by 2 for 2x2 windows); average pooling of floats the plain mean. */
+void qxo_minmax_i64(int64_t n, const int32_t *x, int64_t *mn, int64_t *mx)
+{
+    int64_t lo = n > 0 ? x[0] : 0, hi = lo;
+    for (int64_t i = 1; i < n; ++i) {
+        if (x[i] < lo) lo = x[i];
+        if (x[i] > hi) hi = x[i];
+    }
+    *mn = lo;
+    *mx = hi;
+}
+
+void qxo_minmax_f64(int64_t n, const double *x, double *mn, double *mx)
+{
+    double lo = n > 0 ? x[0] : 0.0, hi = lo;
+    for (int64_t i = 1; i < n; ++i) {
+        if (x[i] < lo) lo = x[i];
+        if (x[i] > hi) hi = x[i];
+    }
+    *mn = lo;
+    *mx = hi;
+}
+
+static inline int64_t floor_div(int64_t a, int64_t b)
+{
+    int64_t q = a / b;
+    if ((a % b != 0) && ((a < 0) != (b < 0))) --q;
+    return q;
+}
+
+void qxo_pool2d_i64(int64_t n, int64_t c, int64_t h, int64_t w, int64_t kh, int64_t kw,
+                    int64_t st, int is_max, const int32_t *x, int64_t *y)
+{
+    const int64_t P = (h - kh) / st + 1, Q = (w - kw) / st + 1;
+#pragma omp parallel for collapse(2) schedule(dynamic, 1)
+    for (int64_t in = 0; in < n; ++in)
+        for (int64_t ic = 0; ic < c; ++ic)
+            for (int64_t p = 0; p < P; ++p)
+                for (int64_t q = 0; q < Q; ++q) {
+                    const int32_t *img = x + (in * c + ic) * h * w;
+                    int64_t acc = is_max ? img[(p * st) * w + q * st] : 0;
+                    for (int64_t r = 0; r < kh; ++r)
+                        for (int64_t s = 0; s < kw; ++s) {
+                            const int64_t v = img[(p * st + r) * w + q * st + s];
+                            if (is_max) acc = v > acc ? v : acc;
+                            else acc += v;
+                        }
+                    y[((in * c + ic) * P + p) * Q + q] = is_max ? acc : floor_div(acc, kh * kw);
+                }
+}
+
+void qxo_pool2d_f64(int64_t n, int64_t c, int64_t h, int64_t w, int64_t kh, int64_t kw,
+                    int64_t st, int is_max, const double *x, double *y)
+{
+    const int64_t P = (h - kh) / st + 1, Q = (w - kw) / st + 1;
+#pragma omp parallel for collapse(2) schedule(dynamic, 1)
+    for (int64_t in = 0; in < n; ++in)
+        for (int64_t ic = 0; ic < c; ++ic)
+            for (int64_t p = 0; p < P; ++p)
+                for (int64_t q = 0; q < Q; ++q) {
+                    const double *img = x + (in * c + ic) * h * w;
+                    double acc = is_max ? img[(p * st) * w + q * st] : 0.0;
+                    for (int64_t r = 0; r < kh; ++r)
+                        for (int64_t s = 0; s < kw; ++s) {
+                            const double v = img[(p * st + r) * w + q * st + s];
+                            if (is_max) acc = v > acc ? v : acc;
+                            else acc += v;
+                        }
+                    y[((in * c + ic) * P + p) * Q + q] = is_max ? acc : acc / (double)(kh * kw);
+                }
 }

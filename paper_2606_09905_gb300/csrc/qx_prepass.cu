@@ -152,6 +152,7 @@ struct ConvPackArgs {
     int *err;
     int x_blocks;          // blocks [0, x_blocks) transpose x; the rest pack w
     int x_tiles_hw, x_tiles_c;
+    int vec_x;             // x rows (one channel of one image) 16-byte aligned
 };
 
 template <typename T, int NX, int NW>
@@ -169,14 +170,24 @@ __global__ void __launch_bounds__(256) pack_conv_kernel(const ConvPackArgs p) {
         const int thw = t % p.x_tiles_hw;
         const int img = t / p.x_tiles_hw;
         const int c0 = tc * 64, hw0 = thw * 64;
-        for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
-            const int cr = i >> 6, pc = i & 63;
-            int32_t v = 0;
-            if (c0 + cr < p.c && hw0 + pc < HW) {
-                v = int32_t(X[(int64_t(img) * p.c + c0 + cr) * HW + hw0 + pc]);
-                p.cx.test(v, p.err);
+        // 8 consecutive pixels of one channel per thread (16-byte loads when
+        // the channel rows allow them)
+        for (int i = threadIdx.x; i < 64 * 8; i += blockDim.x) {
+            const int cr = i >> 3, pg = i & 7;
+            const int hw = hw0 + pg * 8;
+            int32_t v[8];
+            if (c0 + cr < p.c && hw < HW) {
+                const int valid = min(8, HW - hw);
+                load8<T>(X + (int64_t(img) * p.c + c0 + cr) * HW + hw, p.vec_x && valid == 8, valid, v);
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    if (e < valid) p.cx.test(v[e], p.err);
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) v[e] = 0;
             }
-            tile[cr][pc] = v;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) tile[cr][pg * 8 + e] = v[e];
         }
         __syncthreads();
         const int64_t plane_stride = int64_t(p.n) * HW * p.Cp;
@@ -488,6 +499,8 @@ cudaError_t launch_pack_conv(bool i32, const void *x, const void *w, int n, int 
     p.x_tiles_hw = (h * wd + 63) / 64;
     p.x_tiles_c = Cp / 64;
     p.x_blocks = n * p.x_tiles_hw * p.x_tiles_c;
+    const int esz = i32 ? 4 : 2;
+    p.vec_x = (reinterpret_cast<uintptr_t>(x) % 16 == 0) && ((int64_t(h) * wd * esz) % 16 == 0);
     const int64_t w_items = int64_t(k_out) * r * s * (Cp / 8);
     int w_blocks = int((w_items + 255) / 256);
     if (w_blocks > num_sms) w_blocks = num_sms;

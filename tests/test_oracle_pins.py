@@ -243,3 +243,47 @@ def test_fp32_as_written_meets_tolerance_reading():
     ref, _ = oracle.attn_f64(Q, K, V)
     got = ((Q @ K.T) @ V).numpy()
     assert (np.abs(got - ref) <= 1e-5 * oracle.attn_absref(Q, K, V)).all()
+
+
+# ------------------------------------------------ memory-bound operators
+def test_minmax_hand_example_and_numpy(golden):
+    g = golden["minmax_7"]
+    assert oracle.minmax(np.array(g["x"])) == (g["min"], g["max"])
+    rng = np.random.default_rng(7)
+    x = rng.integers(-2**31, 2**31 - 1, size=10007, dtype=np.int64).astype(np.int32)
+    assert oracle.minmax(x) == (int(x.min()), int(x.max()))
+    assert oracle.minmax(x[rng.permutation(x.size)]) == oracle.minmax(x)   # order-free
+    f = rng.standard_normal(999)
+    assert oracle.minmax(f) == (float(f.min()), float(f.max()))
+    assert oracle.minmax(np.full(5, -3)) == (-3, -3)
+
+
+def test_pool_hand_example(golden):
+    g = golden["pool_2x2_s2"]
+    x = np.array(g["x"])
+    assert oracle.pool2d(x, 2, 2, 2, "max").tolist() == g["max"]
+    assert oracle.pool2d(x, 2, 2, 2, "avg").tolist() == g["avg_floor"]
+
+
+@pytest.mark.parametrize("shape,k,s", [((2, 3, 8, 10), 2, 2), ((1, 4, 9, 7), 3, 2), ((2, 2, 6, 6), 2, 1)])
+def test_pool_matches_torch_and_numpy(shape, k, s):
+    rng = np.random.default_rng(sum(shape))
+    x = rng.integers(-1000, 1000, size=shape)
+    xt = torch.from_numpy(x.astype(np.float64))
+    mx = torch.nn.functional.max_pool2d(xt, k, s).numpy()
+    av = torch.nn.functional.avg_pool2d(xt, k, s).numpy() * (k * k)   # window sums
+    assert (oracle.pool2d(x, k, k, s, "max") == mx).all()
+    assert (oracle.pool2d(x, k, k, s, "avg") == np.floor_divide(np.rint(av).astype(np.int64), k * k)).all()
+    f = rng.standard_normal(shape)
+    ft = torch.from_numpy(f)
+    np.testing.assert_allclose(oracle.pool2d(f, k, k, s, "avg"),
+                               torch.nn.functional.avg_pool2d(ft, k, s).numpy(), rtol=0, atol=1e-12)
+    assert (oracle.pool2d(f, k, k, s, "max") == torch.nn.functional.max_pool2d(ft, k, s).numpy()).all()
+
+
+def test_pool_2x2_reshape_identity():
+    # 2x2 / stride 2 max pooling is a reshape-and-reduce
+    x = np.random.default_rng(3).integers(-50, 50, size=(3, 2, 6, 8))
+    ref = x.reshape(3, 2, 3, 2, 4, 2).max(axis=(3, 5))
+    assert (oracle.pool2d(x, 2, 2, 2, "max") == ref).all()
+    assert (oracle.pool2d(np.full((1, 1, 4, 4), -7), 2, 2, 2, "avg") == -7).all()
