@@ -224,12 +224,13 @@ def op_times(torch, make_plan, call, ops, reps, dev):
             "execute_gops": round(ops / (x * 1e-3) / 1e9, 1), "status": st}
 
 
+
 def op_roofline(flops_tensor: float, tensor_peak_tflops: float, hbm_bytes: float,
                 hbm_gbs: float, exec_ms: float) -> dict:
     """Roofline of one operator call: the slower of its tensor work (FLOPs of
     the exact scheme's MMAs at the peak of their kind) and its algorithmic
     bytes (operands read once, output written once) at HBM bandwidth."""
-    t_tensor = flops_tensor / (tensor_peak_tflops * 1e12) * 1e3
+    t_tensor = flops_tensor / (tensor_peak_tflops * 1e12) * 1e3 if flops_tensor else 0.0
     t_hbm = hbm_bytes / (hbm_gbs * 1e9) * 1e3
     bound = "tensor" if t_tensor >= t_hbm else "hbm"
     t_roof = max(t_tensor, t_hbm)
@@ -288,7 +289,47 @@ def operators(torch, qx, inputs, dev, only=None):
         r["roofline"] = op_roofline(flops, tensor_peak, nbytes, peaks["hbm_gbs"], r["execute_ms"])
         return r
 
-    table = {"conv_int16": lambda: conv(qx.I16), "conv_int32": lambda: conv(qx.I32),
+    def stream_op(name, make_desc, make_input, call, in_bytes, out_bytes):
+        x = make_input().to(dev)
+        r = op_times(torch, lambda: qx.Plan(make_desc()), lambda p: call(p, x), 0.0, 50, dev)
+        for k in ("cached_gops", "execute_gops"):
+            r.pop(k)
+        r["execute_gibs"] = round(in_bytes / (r["execute_ms"] * 1e-3) / 2**30, 1)
+        r["cached_gibs"] = round(in_bytes / (r["cached_ms"] * 1e-3) / 2**30, 1)
+        r["roofline"] = op_roofline(0.0, 1.0, in_bytes + out_bytes, peaks["hbm_gbs"], r["execute_ms"])
+        r["workload"] = name
+        return r
+
+    g = torch.Generator().manual_seed(0)
+    n32, n16 = 1 << 28, 1 << 29                 # 1 GiB of input each
+    pool_shape = (32, 128, 112, 112)
+    pool_in = 32 * 128 * 112 * 112 * 4
+
+    def mm(dtype, n):
+        out = torch.empty(2, dtype=torch.int32 if dtype == qx.I32 else torch.int16, device=dev)
+        return lambda p, x: p.minmax(x, out)
+
+    table = {"minmax_int32": lambda: stream_op(
+                 f"min/max of 2^28 int32 (1 GiB)", lambda: qx.minmax_desc(n32, qx.I32),
+                 lambda: torch.randint(-2**31, 2**31 - 1, (n32,), generator=g, dtype=torch.int32),
+                 mm(qx.I32, n32), n32 * 4, 8),
+             "minmax_int16": lambda: stream_op(
+                 f"min/max of 2^29 int16 (1 GiB)", lambda: qx.minmax_desc(n16, qx.I16),
+                 lambda: torch.randint(-2**15, 2**15 - 1, (n16,), generator=g, dtype=torch.int16),
+                 mm(qx.I16, n16), n16 * 2, 4),
+             "avgpool_int32": lambda: stream_op(
+                 "AvgPool 2x2/2 int32, NCHW 32x128x112x112 (floor mean)",
+                 lambda: qx.pool_desc(*pool_shape, 2, 2, 2, "avg", qx.I32),
+                 lambda: torch.randint(-2**20, 2**20, pool_shape, generator=g, dtype=torch.int32),
+                 (lambda p, x, y=torch.empty((32, 128, 56, 56), dtype=torch.int32, device=dev):
+                  p.pool2d(x, y)), pool_in, pool_in // 4),
+             "maxpool_fp32": lambda: stream_op(
+                 "MaxPool 2x2/2 fp32, NCHW 32x128x112x112",
+                 lambda: qx.pool_desc(*pool_shape, 2, 2, 2, "max", qx.F32),
+                 lambda: torch.randn(pool_shape, generator=g),
+                 (lambda p, x, y=torch.empty((32, 128, 56, 56), dtype=torch.float32, device=dev):
+                  p.pool2d(x, y)), pool_in, pool_in // 4),
+             "conv_int16": lambda: conv(qx.I16), "conv_int32": lambda: conv(qx.I32),
              "conv_fp32": lambda: conv(qx.F32), "attn_int16": lambda: attn(qx.I16),
              "attn_int32": lambda: attn(qx.I32), "attn_fp32": lambda: attn(qx.F32)}
     return {k: f() for k, f in table.items() if only is None or k in only}

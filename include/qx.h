@@ -61,7 +61,14 @@ typedef enum {
     QX_ERR_DEVICE = 7        /* no usable sm_103 device                     */
 } qx_status;
 
-typedef enum { QX_OP_GEMM = 0, QX_OP_CONV2D = 1, QX_OP_ATTN = 2 } qx_op;
+typedef enum {
+    QX_OP_GEMM = 0,
+    QX_OP_CONV2D = 1,
+    QX_OP_ATTN = 2,
+    QX_OP_MINMAX = 3,   /* memory-bound operators of Table 2 */
+    QX_OP_MAXPOOL = 4,
+    QX_OP_AVGPOOL = 5
+} qx_op;
 typedef enum { QX_I16 = 0, QX_I32 = 1, QX_F32 = 2 } qx_dtype;
 
 /* Inclusive operand-range contract (Methodology: operand-range contracts
@@ -85,6 +92,9 @@ typedef struct {
     int64_t n, c, h, w, k_out, r, s, stride, pad;
     /* Attention core: Q, K, V and O are L x d, row-major, tightly packed. */
     int64_t L, d;
+    /* Min/max: M is the element count.  Pooling: n, c, h, w give the NCHW
+     * input, r x s the window and stride its step; pad must be 0; the output
+     * is NCHW (n, c, P, Q), P = (h - r) / stride + 1, Q likewise. */
     /* Ranges.  GEMM: range_a = A, range_b = B.  Conv2D: range_a = x,
      * range_b = weights.  Attention: range_a = Q, range_b = K, range_c = V.
      * Ignored for F32. */
@@ -164,6 +174,20 @@ qx_status qx_attn_core(qx_plan plan, const void *Q, const void *K,
 qx_status qx_pack(qx_plan plan, const void *a, const void *b, const void *c,
                   qx_stream stream);
 qx_status qx_run_packed(qx_plan plan, void *out, qx_stream stream);
+
+/* Min/max reduction (Table 2 min/max rows): result[0] = smallest and
+ * result[1] = largest of the M elements of x; x and result (a device buffer
+ * of two elements) have the plan's in_dtype (I16, I32 or F32; NaNs give an
+ * unspecified result).  Plan op MINMAX.  The plan's workspace holds the
+ * per-block partial results. */
+qx_status qx_minmax(qx_plan plan, const void *x, void *result, qx_stream stream);
+
+/* 2-D pooling without padding (Table 2 pooling rows): plan op MAXPOOL takes
+ * the window maximum; AVGPOOL the window mean, floor(sum / (r * s)) for
+ * integers (an arithmetic shift by 2 for the paper's 2x2 windows) and the
+ * FP32 mean for floats.  x and y are NCHW of the plan's in_dtype (I16, I32
+ * or F32). */
+qx_status qx_pool2d(qx_plan plan, const void *x, void *y, qx_stream stream);
 
 /* Synchronises the plan's device, then returns and clears the sticky device
  * error word (QX_ERR_TIMEOUT or QX_ERR_CONTRACT), or QX_OK. */

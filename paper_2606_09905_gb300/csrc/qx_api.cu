@@ -38,6 +38,11 @@ cudaError_t launch_pack_conv_f32(const float *x, const float *w, int n, int c, i
                                  int k_out, int r, int s, int Cp, float *x_planes, float *w_planes,
                                  int num_sms, cudaStream_t st);
 cudaError_t attn_prepare();
+int minmax_blocks(int num_sms);
+cudaError_t launch_minmax(int dtype, const void *x, int64_t n, void *result, void *partial,
+                          unsigned *counter, int num_sms, cudaStream_t st);
+cudaError_t launch_pool2d(int dtype, bool is_max, const void *x, void *y, int n, int c, int h, int w,
+                          int kh, int kw, int stride, int num_sms, cudaStream_t st);
 cudaError_t attn_f32_prepare();
 cudaError_t attn_f32_launch(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_pack_attn_f32(const float *Q, const float *K, const float *V, int L, int d, int Lp,
@@ -305,6 +310,20 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
             if (max_keys) *max_keys = int(std::min<int64_t>(best_keys, INT32_MAX / 2));
             return QX_OK;
         }
+        case QX_OP_MINMAX:
+            if (d->M < 1) return fail(QX_ERR_INVALID_ARG, "min/max needs M >= 1 elements");
+            *count = 0;
+            return QX_OK;
+        case QX_OP_MAXPOOL:
+        case QX_OP_AVGPOOL:
+            if (d->n < 1 || d->c < 1 || d->r < 1 || d->s < 1 || d->stride < 1 || d->h < d->r ||
+                d->w < d->s)
+                return fail(QX_ERR_INVALID_ARG, "pooling sizes out of range");
+            if (d->pad != 0) return fail(QX_ERR_UNSUPPORTED, "pooling with padding");
+            if (d->n * d->c * d->h * d->w > (int64_t(1) << 40))
+                return fail(QX_ERR_UNSUPPORTED, "pooling input too large");
+            *count = 0;
+            return QX_OK;
         default:
             return fail(QX_ERR_INVALID_ARG, "unknown op %d", int(d->op));
     }
@@ -644,6 +663,18 @@ static qx_status build_attn(qx_plan p) {
     return QX_OK;
 }
 
+// Min/max and pooling: no packing; min/max keeps its per-block partials and
+// an arrival counter (zeroed here, rearmed by every call) in the workspace.
+static qx_status build_stream_op(qx_plan p) {
+    size_t bytes = 256;
+    if (p->desc.op == QX_OP_MINMAX) bytes += 256 + align256(size_t(minmax_blocks(p->num_sms)) * 2 * 8);
+    p->ws_bytes = bytes;
+    QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
+    QX_CUDA(cudaMemset(p->ws, 0, p->ws_bytes), "workspace reset");
+    p->err = static_cast<int *>(p->ws);
+    return QX_OK;
+}
+
 // ================================================================ C ABI
 extern "C" {
 
@@ -714,6 +745,9 @@ qx_status qx_plan_create(const qx_plan_desc *desc, int device, qx_plan *out) {
         case QX_OP_GEMM: st = build_gemm(p); break;
         case QX_OP_CONV2D: st = build_conv(p); break;
         case QX_OP_ATTN: st = build_attn(p); break;
+        case QX_OP_MINMAX:
+        case QX_OP_MAXPOOL:
+        case QX_OP_AVGPOOL: st = build_stream_op(p); break;
         default: st = fail(QX_ERR_INVALID_ARG, "unknown op");
     }
     if (st != QX_OK) {
@@ -762,12 +796,20 @@ qx_status qx_plan_status(qx_plan p) {
 static bool aligned16(const void *ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
 
 static const char *op_name(qx_op op) {
-    return op == QX_OP_GEMM ? "GEMM" : op == QX_OP_CONV2D ? "conv" : "attention";
+    switch (op) {
+        case QX_OP_GEMM: return "GEMM";
+        case QX_OP_CONV2D: return "conv";
+        case QX_OP_ATTN: return "attention";
+        case QX_OP_MINMAX: return "min/max";
+        default: return "pooling";
+    }
 }
 
 // Operand packing: operands -> FP16 limb planes in the workspace.
 static qx_status pack(qx_plan p, const void *a, const void *b, const void *c, cudaStream_t st) {
     const qx_plan_desc &d = p->desc;
+    if (d.op == QX_OP_MINMAX || d.op == QX_OP_MAXPOOL || d.op == QX_OP_AVGPOOL)
+        return fail(QX_ERR_INVALID_ARG, "min/max and pooling plans have no packing step");
     const int check = (d.flags & QX_FLAG_CHECK_RANGES) ? 1 : 0;
     const bool i32 = d.in_dtype == QX_I32;
     switch (d.op) {
@@ -828,6 +870,8 @@ static qx_status pack(qx_plan p, const void *a, const void *b, const void *c, cu
 // The tensor-core kernel on the packed workspace.
 static qx_status run_packed(qx_plan p, void *out, cudaStream_t st) {
     const qx_plan_desc &d = p->desc;
+    if (d.op == QX_OP_MINMAX || d.op == QX_OP_MAXPOOL || d.op == QX_OP_AVGPOOL)
+        return fail(QX_ERR_INVALID_ARG, "min/max and pooling plans have no packing step");
     if (!out) return fail(QX_ERR_INVALID_ARG, "null output");
     if (!aligned16(out)) return fail(QX_ERR_UNSUPPORTED, "output must be 16-byte aligned");
     switch (d.op) {
@@ -902,6 +946,41 @@ qx_status qx_conv2d_gemm(qx_plan p, const void *x, const void *w, void *y, qx_st
 qx_status qx_attn_core(qx_plan p, const void *Q, const void *K, const void *V, void *O,
                        qx_stream stream) {
     return execute(p, QX_OP_ATTN, QX_I16, Q, K, V, O, stream);
+}
+
+qx_status qx_minmax(qx_plan p, const void *x, void *result, qx_stream stream) {
+    if (!p) return fail(QX_ERR_INVALID_ARG, "null plan");
+    const qx_plan_desc &d = p->desc;
+    if (d.op != QX_OP_MINMAX) return fail(QX_ERR_INVALID_ARG, "plan is not a min/max plan");
+    if (!x || !result) return fail(QX_ERR_INVALID_ARG, "null operand");
+    const size_t esz = d.in_dtype == QX_I16 ? 2 : 4;
+    if ((reinterpret_cast<uintptr_t>(x) % esz) || (reinterpret_cast<uintptr_t>(result) % esz))
+        return fail(QX_ERR_UNSUPPORTED, "operands must be aligned to their element size");
+    DeviceScope scope;
+    QX_CUDA(scope.enter(p->device), "cudaSetDevice");
+    char *ws = static_cast<char *>(p->ws);
+    QX_CUDA(launch_minmax(d.in_dtype, x, d.M, result, ws + 512, reinterpret_cast<unsigned *>(ws + 256),
+                          p->num_sms, reinterpret_cast<cudaStream_t>(stream)),
+            "min/max launch");
+    return QX_OK;
+}
+
+qx_status qx_pool2d(qx_plan p, const void *x, void *y, qx_stream stream) {
+    if (!p) return fail(QX_ERR_INVALID_ARG, "null plan");
+    const qx_plan_desc &d = p->desc;
+    if (d.op != QX_OP_MAXPOOL && d.op != QX_OP_AVGPOOL)
+        return fail(QX_ERR_INVALID_ARG, "plan is not a pooling plan");
+    if (!x || !y) return fail(QX_ERR_INVALID_ARG, "null operand");
+    const size_t esz = d.in_dtype == QX_I16 ? 2 : 4;
+    if ((reinterpret_cast<uintptr_t>(x) % esz) || (reinterpret_cast<uintptr_t>(y) % esz))
+        return fail(QX_ERR_UNSUPPORTED, "operands must be aligned to their element size");
+    DeviceScope scope;
+    QX_CUDA(scope.enter(p->device), "cudaSetDevice");
+    QX_CUDA(launch_pool2d(d.in_dtype, d.op == QX_OP_MAXPOOL, x, y, int(d.n), int(d.c), int(d.h),
+                          int(d.w), int(d.r), int(d.s), int(d.stride), p->num_sms,
+                          reinterpret_cast<cudaStream_t>(stream)),
+            "pooling launch");
+    return QX_OK;
 }
 
 qx_status qx_pack(qx_plan p, const void *a, const void *b, const void *c, qx_stream stream) {

@@ -20,7 +20,7 @@ LIB_PATH = os.path.join(_HERE, "libqx.so")
 # qx_status
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CONTRACT, ERR_OOM, ERR_CUDA, ERR_TIMEOUT, ERR_DEVICE = range(8)
 # qx_op / qx_dtype
-OP_GEMM, OP_CONV2D, OP_ATTN = 0, 1, 2
+OP_GEMM, OP_CONV2D, OP_ATTN, OP_MINMAX, OP_MAXPOOL, OP_AVGPOOL = 0, 1, 2, 3, 4, 5
 I16, I32, F32 = 0, 1, 2
 FLAG_CHECK_RANGES = 1
 
@@ -28,7 +28,8 @@ FLAG_CHECK_RANGES = 1
 EXPORTS = ("qx_plan_create", "qx_plan_destroy", "qx_plan_query", "qx_plan_info",
            "qx_gemm_i16_i32", "qx_gemm_i32", "qx_conv2d_gemm", "qx_attn_core",
            "qx_pack", "qx_run_packed", "qx_plan_status", "qx_status_string",
-           "qx_last_error", "qx_version", "qx_gemm_i16_i32_noalloc")
+           "qx_last_error", "qx_version", "qx_gemm_i16_i32_noalloc", "qx_minmax",
+           "qx_pool2d")
 
 
 class QxError(RuntimeError):
@@ -94,6 +95,8 @@ def load() -> ctypes.CDLL:
             "qx_status_string": ([ctypes.c_int], ctypes.c_char_p),
             "qx_last_error": ([], ctypes.c_char_p),
             "qx_version": ([], ctypes.c_int),
+            "qx_minmax": ([P, V, V, V], ctypes.c_int),
+            "qx_pool2d": ([P, V, V, V], ctypes.c_int),
             "qx_gemm_i16_i32_noalloc": ([ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, Range,
                                          Range, ctypes.c_uint, V, V, V, V, V], ctypes.c_int),
         }
@@ -131,6 +134,17 @@ def conv_desc(n, c, h, w, k_out, r, s, stride, pad, range_x, range_w, dtype=I16,
 def attn_desc(L, d, range_q, range_k, range_v, dtype=I16, flags=0) -> PlanDesc:
     return PlanDesc(op=OP_ATTN, in_dtype=dtype, L=L, d=d, range_a=_rng(range_q),
                     range_b=_rng(range_k), range_c=_rng(range_v), flags=flags)
+
+
+def minmax_desc(count, dtype=I32) -> PlanDesc:
+    return PlanDesc(op=OP_MINMAX, in_dtype=dtype, M=count)
+
+
+def pool_desc(n, c, h, w, kh=2, kw=2, stride=2, mode="max", dtype=I32) -> PlanDesc:
+    if mode not in ("max", "avg"):
+        raise ValueError("mode is 'max' or 'avg'")
+    return PlanDesc(op=OP_MAXPOOL if mode == "max" else OP_AVGPOOL, in_dtype=dtype, n=n, c=c, h=h,
+                    w=w, r=kh, s=kw, stride=stride)
 
 
 def query(desc: PlanDesc) -> list[dict]:
@@ -268,6 +282,32 @@ class Plan:
         pw = _ptr(w, dt, (d.k_out, d.c, d.r, d.s), "w")
         py = _ptr(y, out_dt, (d.n, d.k_out, P, Q), "y")
         _check(load().qx_conv2d_gemm(self.handle, px, pw, py, _stream(stream)), "qx_conv2d_gemm")
+        return y
+
+    # -- min/max and pooling ------------------------------------------------
+    def minmax(self, x, out=None, stream=None):
+        """Device tensor [min, max] of the plan's M elements of x."""
+        d = self.desc
+        dt = _TORCH_DT[d.in_dtype]
+        if out is None:
+            out = torch.empty(2, dtype=dt, device=x.device)
+        if not x.is_contiguous() or x.numel() != d.M:
+            raise ValueError(f"x must be contiguous with {d.M} elements")
+        px = _ptr(x, dt, None, "x")
+        po = _ptr(out, dt, (2,), "out")
+        _check(load().qx_minmax(self.handle, px, po, _stream(stream)), "qx_minmax")
+        return out
+
+    def pool2d(self, x, y=None, stream=None):
+        d = self.desc
+        dt = _TORCH_DT[d.in_dtype]
+        P = (d.h - d.r) // d.stride + 1
+        Q = (d.w - d.s) // d.stride + 1
+        if y is None:
+            y = torch.empty((d.n, d.c, P, Q), dtype=dt, device=x.device)
+        px = _ptr(x, dt, (d.n, d.c, d.h, d.w), "x")
+        py = _ptr(y, dt, (d.n, d.c, P, Q), "y")
+        _check(load().qx_pool2d(self.handle, px, py, _stream(stream)), "qx_pool2d")
         return y
 
     # -- attention ----------------------------------------------------------
