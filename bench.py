@@ -244,7 +244,6 @@ def operators(torch, qx, inputs, dev, only=None):
     peaks = load_peaks()
     conv_shape = (8, 64, 56, 56, 128, 3, 3)
     conv_ops = 2.0 * 8 * 128 * 56 * 56 * 64 * 9
-    attn_ops = 4.0 * 1024 * 1024 * 64
 
     def conv(dtype):
         if dtype == qx.F32:
@@ -267,20 +266,22 @@ def operators(torch, qx, inputs, dev, only=None):
         r["roofline"] = op_roofline(m * conv_ops, tensor_peak, nbytes, peaks["hbm_gbs"], r["execute_ms"])
         return r
 
-    def attn(dtype):
+    def attn(dtype, H=0, L=1024, d=64):
+        # H = 0: the paper's single-head core; H >= 1: that many independent heads
+        attn_ops = 4.0 * max(1, H) * L * L * d
         if dtype == qx.F32:
-            Q, K, V = inputs.attn_case_f32(1024, 64, seed=0)
+            Q, K, V = inputs.attn_case_f32(L, d, seed=0, heads=H)
             rng, desc = (0, 0), "fp32 N(0,1), 3xTF32"
         else:
             tdt = torch.int16 if dtype == qx.I16 else torch.int32
-            Q, K, V = inputs.attn_case(1024, 64, -7, 7, seed=0, dtype=tdt)
+            Q, K, V = inputs.attn_case(L, d, -7, 7, seed=0, dtype=tdt, heads=H)
             rng, desc = (-7, 7), f"{'int16' if dtype == qx.I16 else 'int32'} in [-7,7]"
         Q, K, V = Q.to(dev), K.to(dev), V.to(dev)
-        O = torch.empty((1024, 64), dtype=torch.float32 if dtype == qx.F32 else torch.int32,
-                        device=dev)
-        plan_desc = qx.attn_desc(1024, 64, rng, rng, rng, dtype=dtype)
+        O = torch.empty(Q.shape, dtype=torch.float32 if dtype == qx.F32 else torch.int32, device=dev)
+        plan_desc = qx.attn_desc(L, d, rng, rng, rng, dtype=dtype, heads=max(1, H))
         r = op_times(torch, lambda: qx.Plan(plan_desc), lambda p: p.attn(Q, K, V, O), attn_ops, 50, dev)
-        r["workload"] = f"Q,K,V 1024x64, O=(QK^T)V, no softmax, {desc}"
+        shape = f"{L}x{d}" if H == 0 else f"{H} heads x {L}x{d}"
+        r["workload"] = f"Q,K,V {shape}, O=(QK^T)V, no softmax, {desc}"
         s0, s1 = qx.query(plan_desc)
         flops = (s0["mma_per_kstep"] + s1["mma_per_kstep"]) * attn_ops / 2.0
         esz = Q.element_size()
@@ -331,7 +332,9 @@ def operators(torch, qx, inputs, dev, only=None):
                   p.pool2d(x, y)), pool_in, pool_in // 4),
              "conv_int16": lambda: conv(qx.I16), "conv_int32": lambda: conv(qx.I32),
              "conv_fp32": lambda: conv(qx.F32), "attn_int16": lambda: attn(qx.I16),
-             "attn_int32": lambda: attn(qx.I32), "attn_fp32": lambda: attn(qx.F32)}
+             "attn_int32": lambda: attn(qx.I32), "attn_fp32": lambda: attn(qx.F32),
+             "attn_mh_int16": lambda: attn(qx.I16, H=32, L=2048),
+             "attn_mh_fp32": lambda: attn(qx.F32, H=32, L=2048)}
     return {k: f() for k, f in table.items() if only is None or k in only}
 
 

@@ -90,7 +90,8 @@ typedef struct {
      * NCHW (n, k_out, P, Q), P = (h + 2 pad - r) / stride + 1, Q likewise;
      * cross-correlation, zero padding, no bias, all tightly packed. */
     int64_t n, c, h, w, k_out, r, s, stride, pad;
-    /* Attention core: Q, K, V and O are L x d, row-major, tightly packed. */
+    /* Attention core: Q, K, V and O are heads x L x d, row-major, tightly
+     * packed (see `heads` below). */
     int64_t L, d;
     /* Min/max: M is the element count.  Pooling: n, c, h, w give the NCHW
      * input, r x s the window and stride its step; pad must be 0; the output
@@ -100,6 +101,10 @@ typedef struct {
      * Ignored for F32. */
     qx_range range_a, range_b, range_c;
     unsigned flags;
+    /* Attention: number of independent heads (batched cores) sharing L, d
+     * and the range contract; head h reads Q[h], K[h], V[h] and writes O[h].
+     * 0 and 1 both mean a single head.  At most 65535.  Ignored otherwise. */
+    int64_t heads;
 } qx_plan_desc;
 
 /* How the plan makes one contraction exact on FP16 tensor cores.  An
@@ -156,10 +161,12 @@ qx_status qx_gemm_i32(qx_plan plan, const int32_t *A, const int32_t *B,
 qx_status qx_conv2d_gemm(qx_plan plan, const void *x, const void *w, void *y,
                          qx_stream stream);
 
-/* Single-head attention core O = (Q K^T) V, no softmax, no scale
- * (Methodology; Table 2).  Q, K, V, O as in qx_plan_desc, element type per
- * in_dtype (O is int32 for integer plans, float for F32).  S = Q K^T is
- * kept on chip; it never goes to device memory. */
+/* Attention core O = (Q K^T) V, no softmax, no scale (Methodology; Table 2:
+ * the paper's single-head core).  A plan with heads > 1 runs that many
+ * independent cores in one launch, O[h] = (Q[h] K[h]^T) V[h].  Q, K, V, O as
+ * in qx_plan_desc, element type per in_dtype (O is int32 for integer plans,
+ * float for F32).  S = Q K^T is kept on chip; it never goes to device
+ * memory. */
 qx_status qx_attn_core(qx_plan plan, const void *Q, const void *K,
                        const void *V, void *O, qx_stream stream);
 

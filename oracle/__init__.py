@@ -15,7 +15,8 @@ Definitions (paper: Abstract, Methodology paragraph, Table 1, Table 2):
 * ``gemm``    C = A B, int64, plus the largest |partial sum| in k order (the
   accumulation contract of the Methodology paragraph).
 * ``conv2d``  direct NCHW/KCRS cross-correlation with zero padding, no bias.
-* ``attn``    S = Q K^T then O = S V, no softmax and no scale.
+* ``attn``    S = Q K^T then O = S V, no softmax and no scale; given (heads,
+  L, d) operands, the same core independently for every head.
 * ``minmax``  smallest and largest element (Table 2 min/max rows).
 * ``pool2d``  NCHW max / average pooling without padding (Table 2 pooling
   rows); integer averages are floor(window sum / window size).
@@ -188,8 +189,22 @@ def _attn_shapes(Q, K, V):
     return Q.shape
 
 
+def _per_head(fn, Q, K, V):
+    """Batched cores: ``fn`` on every head of (heads, L, d) operands; the
+    results are stacked along a new leading axis (scalars: the maximum)."""
+    Q, K, V = _np(Q), _np(K), _np(V)
+    if Q.ndim != 3 or Q.shape != K.shape or Q.shape != V.shape:
+        raise ValueError(f"attention shapes {Q.shape} {K.shape} {V.shape}")
+    outs = [fn(Q[h], K[h], V[h]) for h in range(Q.shape[0])]
+    return tuple(max(col) if isinstance(col[0], int) else np.stack(col) for col in zip(*outs))
+
+
 def attn(Q, K, V):
-    """Exact O = (Q K^T) V as written.  Returns ``(O, S, max_abs_S)``."""
+    """Exact O = (Q K^T) V as written.  Returns ``(O, S, max_abs_S)``.
+    (heads, L, d) operands give (heads, L, d) O, (heads, L, L) S and the
+    largest |S| over all heads."""
+    if _np(Q).ndim == 3:
+        return _per_head(attn, Q, K, V)
     Q = _as_i32(Q)
     K = _as_i32(K)
     V = _as_i32(V)
@@ -203,6 +218,8 @@ def attn(Q, K, V):
 
 
 def attn_f64(Q, K, V):
+    if _np(Q).ndim == 3:
+        return _per_head(attn_f64, Q, K, V)
     Q = _as_f64(Q)
     K = _as_f64(K)
     V = _as_f64(V)

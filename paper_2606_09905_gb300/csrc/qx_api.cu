@@ -45,8 +45,8 @@ cudaError_t launch_pool2d(int dtype, bool is_max, const void *x, void *y, int n,
                           int kh, int kw, int stride, int num_sms, cudaStream_t st);
 cudaError_t attn_f32_prepare();
 cudaError_t attn_f32_launch(const AttnArgs &a, cudaStream_t stream);
-cudaError_t launch_pack_attn_f32(const float *Q, const float *K, const float *V, int L, int d, int Lp,
-                                 float *q, float *k, float *vt, int num_sms, cudaStream_t st);
+cudaError_t launch_pack_attn_f32(const float *Q, const float *K, const float *V, int heads, int L, int d,
+                                 int Lp, float *q, float *k, float *vt, int num_sms, cudaStream_t st);
 int attn_max_cluster();
 cudaError_t attn_launch(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_pack_gemm(bool i32, const void *A, const void *B, int64_t lda, int64_t ldb,
@@ -57,7 +57,7 @@ cudaError_t launch_pack_conv(bool i32, const void *x, const void *w, int n, int 
                              int k_out, int r, int s, int Cp, __half *x_planes, __half *w_planes,
                              int nx, int shift_x, int nw, int shift_w, int check, qx_range rx,
                              qx_range rw, int *err, int num_sms, cudaStream_t st);
-cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int L, int d,
+cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int heads, int L, int d,
                              int dp, int Lp, __half *q, __half *k, __half *vt, int int_check,
                              qx_range rq, qx_range rk, qx_range rv, int *err, int num_sms,
                              cudaStream_t st);
@@ -240,8 +240,11 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
             return QX_OK;
         }
         case QX_OP_ATTN: {
-            if (d->L < 1 || d->d < 1 || d->L > (1 << 24))
+            if (d->L < 1 || d->d < 1 || d->L > (1 << 24) || d->heads < 0)
                 return fail(QX_ERR_INVALID_ARG, "attention sizes out of range");
+            if (d->heads > 65535) return fail(QX_ERR_UNSUPPORTED, "more than 65535 heads");
+            if (std::max<int64_t>(1, d->heads) * d->L > (int64_t(1) << 31) - 1)
+                return fail(QX_ERR_UNSUPPORTED, "heads * L above 2^31 - 1");
             if (d->d > 128) return fail(QX_ERR_UNSUPPORTED, "attention head size above 128");
             if (f32) {
                 if (d->d > 64) return fail(QX_ERR_UNSUPPORTED, "FP32 attention head size above 64");
@@ -562,19 +565,22 @@ static void attn_splits(int key_blocks, int q_tiles, int num_sms, int max_blocks
 
 static qx_status build_attn_f32(qx_plan p) {
     const qx_plan_desc &d = p->desc;
+    const uint64_t H = uint64_t(d.heads);
     p->dp = 64;
     p->Lp = int((d.L + 7) / 8 * 8);
     AttnArgs &a = p->attn;
     memset(&a, 0, sizeof a);
     a.L = int(d.L);
     a.d = int(d.d);
+    a.heads = int(d.heads);
     a.q_tiles = int((d.L + 127) / 128);
     int splits = 1, per = 1;
-    attn_splits(int((d.L + 31) / 32), a.q_tiles, p->num_sms, INT32_MAX, &splits, &per);
+    attn_splits(int((d.L + 31) / 32), a.q_tiles * a.heads, p->num_sms, INT32_MAX, &splits, &per);
     a.key_splits = splits;
     a.keys_per_split = per * 32;
-    const size_t qk_bytes = size_t(2) * d.L * 64 * 4;
-    const size_t vt_bytes = size_t(2) * 64 * p->Lp * 4;
+    // planes [head][big/small][L][64] and [head][big/small][64][Lp]
+    const size_t qk_bytes = size_t(H) * 2 * d.L * 64 * 4;
+    const size_t vt_bytes = size_t(H) * 2 * 64 * p->Lp * 4;
     p->ws_bytes = 256 + 2 * align256(qk_bytes) + align256(vt_bytes);
     QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
     char *base = static_cast<char *>(p->ws);
@@ -587,7 +593,7 @@ static qx_status build_attn_f32(qx_plan p) {
     p->fvt = reinterpret_cast<float *>(base + off);
     QX_CUDA(cudaMemset(p->ws, 0, p->ws_bytes), "workspace reset");
     {
-        const uint64_t dims[3] = {64, uint64_t(d.L), 2};
+        const uint64_t dims[3] = {64, uint64_t(d.L), 2 * H};
         const uint64_t str[2] = {64 * 4, uint64_t(d.L) * 64 * 4};
         const uint32_t boxq[3] = {32, 128, 2};
         const uint32_t boxk[3] = {32, 32, 2};
@@ -597,7 +603,7 @@ static qx_status build_attn_f32(qx_plan p) {
         if (st != QX_OK) return st;
     }
     {
-        const uint64_t dims[3] = {uint64_t(d.L), 64, 2};
+        const uint64_t dims[3] = {uint64_t(d.L), 64, 2 * H};
         const uint64_t str[2] = {uint64_t(p->Lp) * 4, uint64_t(64) * p->Lp * 4};
         const uint32_t box[3] = {32, 128, 2};
         qx_status st = encode_tiled(&a.tm_vt, p->fvt, 3, dims, str, box, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
@@ -611,10 +617,12 @@ static qx_status build_attn_f32(qx_plan p) {
 static qx_status build_attn(qx_plan p) {
     const qx_plan_desc &d = p->desc;
     if (d.in_dtype == QX_F32) return build_attn_f32(p);
+    const uint64_t H = uint64_t(d.heads);
     p->dp = d.d <= 64 ? 64 : 128;
     p->Lp = int((d.L + 7) / 8 * 8);
-    const size_t qk_bytes = size_t(d.L) * p->dp * 2;
-    const size_t vt_bytes = size_t(p->dp) * p->Lp * 2;
+    // Q, K: [head][L][dp]; V^T: [head][dp][Lp]
+    const size_t qk_bytes = size_t(H) * d.L * p->dp * 2;
+    const size_t vt_bytes = size_t(H) * p->dp * p->Lp * 2;
     p->ws_bytes = 256 + 2 * align256(qk_bytes) + align256(vt_bytes);
     QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
     char *base = static_cast<char *>(p->ws);
@@ -627,30 +635,37 @@ static qx_status build_attn(qx_plan p) {
     AttnArgs &a = p->attn;
     memset(&a, 0, sizeof a);
     {
-        const uint64_t dims[2] = {uint64_t(p->dp), uint64_t(d.L)};
-        const uint64_t str[1] = {uint64_t(p->dp) * 2};
-        const uint32_t boxq[2] = {64, 128};
-        const uint32_t boxk[2] = {64, 64};
-        qx_status st = encode_tiled(&a.tm_q, p->aq, 2, dims, str, boxq);
+        const uint64_t dims[3] = {uint64_t(p->dp), uint64_t(d.L), H};
+        const uint64_t str[2] = {uint64_t(p->dp) * 2, uint64_t(d.L) * p->dp * 2};
+        const uint32_t boxq[3] = {64, 128, 1};   // 128 queries
+        const uint32_t boxk[3] = {64, 128, 1};   // 128 keys
+        qx_status st = encode_tiled(&a.tm_q, p->aq, 3, dims, str, boxq);
         if (st != QX_OK) return st;
-        st = encode_tiled(&a.tm_k, p->ak, 2, dims, str, boxk);
+        st = encode_tiled(&a.tm_k, p->ak, 3, dims, str, boxk);
         if (st != QX_OK) return st;
     }
     {
-        const uint64_t dims[2] = {uint64_t(d.L), uint64_t(p->dp)};
-        const uint64_t str[1] = {uint64_t(p->Lp) * 2};
-        const uint32_t box[2] = {64, 128};
-        qx_status st = encode_tiled(&a.tm_vt, p->avt, 2, dims, str, box);
+        const uint64_t dims[3] = {uint64_t(d.L), uint64_t(p->dp), H};
+        const uint64_t str[2] = {uint64_t(p->Lp) * 2, uint64_t(p->dp) * p->Lp * 2};
+        const uint32_t box[3] = {64, uint32_t(p->dp), 1};
+        qx_status st = encode_tiled(&a.tm_vt, p->avt, 3, dims, str, box);
         if (st != QX_OK) return st;
     }
     a.err = p->err;
     a.L = int(d.L);
     a.d = int(d.d);
+    a.heads = int(d.heads);
     a.q_tiles = int((d.L + 127) / 128);
+    // splits are whole 64-key granules; the kernel walks 128-key blocks and
+    // masks keys past the end of its run, so an even count wastes nothing
     const int key_blocks = int((d.L + 63) / 64);
     const int max_blocks = std::max(1, p->max_keys / 64);
     int splits = 1, per = 1;
-    attn_splits(key_blocks, a.q_tiles, p->num_sms, max_blocks, &splits, &per);
+    attn_splits(key_blocks, a.q_tiles * a.heads, p->num_sms, max_blocks, &splits, &per);
+    if ((per & 1) && per + 1 <= max_blocks && per < key_blocks) {
+        ++per;
+        splits = (key_blocks + per - 1) / per;
+    }
     if (per > max_blocks)
         return fail(QX_ERR_UNSUPPORTED,
                     "L = %lld needs more than %d exact key chunks per query tile",
@@ -712,6 +727,7 @@ qx_status qx_plan_create(const qx_plan_desc *desc, int device, qx_plan *out) {
     *out = nullptr;
     if (!desc) return fail(QX_ERR_INVALID_ARG, "null descriptor");
     qx_plan_desc d = *desc;
+    if (d.op == QX_OP_ATTN && d.heads == 0) d.heads = 1;
     if (d.op == QX_OP_GEMM) {
         if (d.lda == 0) d.lda = d.K;
         if (d.ldb == 0) d.ldb = d.N;
@@ -852,12 +868,12 @@ static qx_status pack(qx_plan p, const void *a, const void *b, const void *c, cu
             if (d.in_dtype == QX_F32) {
                 QX_CUDA(launch_pack_attn_f32(static_cast<const float *>(a),
                                              static_cast<const float *>(b),
-                                             static_cast<const float *>(c), int(d.L), int(d.d),
-                                             p->Lp, p->fq, p->fk, p->fvt, p->num_sms, st),
+                                             static_cast<const float *>(c), int(d.heads), int(d.L),
+                                             int(d.d), p->Lp, p->fq, p->fk, p->fvt, p->num_sms, st),
                         "operand packing launch");
                 return QX_OK;
             }
-            QX_CUDA(launch_pack_attn(i32, a, b, c, int(d.L), int(d.d), p->dp, p->Lp, p->aq, p->ak,
+            QX_CUDA(launch_pack_attn(i32, a, b, c, int(d.heads), int(d.L), int(d.d), p->dp, p->Lp, p->aq, p->ak,
                                      p->avt, check, d.range_a, d.range_b, d.range_c, p->err,
                                      p->num_sms, st),
                     "operand packing launch");

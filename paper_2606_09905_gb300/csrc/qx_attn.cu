@@ -1,25 +1,28 @@
-// qx_attn.cu -- the single-head attention core O = (Q K^T) V, no softmax and
-// no scale (paper: Methodology; Table 2 attention rows), as two chained
-// products on the tiled substrate with S = Q K^T kept on chip.
+// qx_attn.cu -- the attention core O = (Q K^T) V, no softmax and no scale
+// (paper: Methodology; Table 2 attention rows), as two chained products on
+// the tiled substrate with S = Q K^T kept on chip.
 //
-// Grid: query tiles (128 queries) x key splits; the splits of one query tile
-// form one thread-block cluster.  Each CTA walks its run of key blocks:
+// Grid: x = query tiles (128 queries) x key splits, y = heads.  The splits of
+// one query tile form one thread-block cluster; heads are independent cores
+// (their packed operands are the outer dimension of every tensor map, so a
+// tile never reaches into the next head).  Each CTA walks its run of key
+// blocks:
 //   1. S_b = Q K_b^T        tcgen05 into TMEM (M = 128 queries, N = keys);
-//   2. S_b -> operand       each thread reads its query row of S from TMEM and
-//                           writes it back to shared memory as the operand of
-//                           the second product (K-major, 128B-swizzled);
-//   3. O^T += V_b^T S_b^T   tcgen05 into TMEM (M = 128 rows of V^T, i.e. the d
-//                           outputs padded with zeros; N = 2 x 128 queries).
+//   2. S_b -> operand       threads read query rows of S from TMEM and write
+//                           them back to shared memory as the A operand of the
+//                           second product (K-major, 128B-swizzled);
+//   3. O += S_b V_b         tcgen05 into TMEM (integer kind: M = 128 queries,
+//                           N = head size; FP32 kind: O^T += V_b^T S_b^T).
 // At the end every CTA leaves its partial O in its own shared memory; after a
 // cluster barrier, CTA r of the cluster adds slice r of the query rows over
 // all CTAs of the cluster (distributed shared memory, fixed rank order) and
 // writes O.  No atomics, no zeroing, and the same order on every run.
 //
 // Integer kind (FP16 digits, exact): S is exact because the plan bounds
-// d * max|Q| * max|K| by 2^24; S is split into two balanced digits (rows
-// 0-127 low, 128-255 high of the N-side tile) and the plan bounds
-// keys-per-CTA * max|digit| * max|V| by 2^24, so O^T's FP32 sums are exact;
-// O = lo + (hi << shift) in wrapping int32.
+// d * max|Q| * max|K| by 2^24; S is split into two balanced digits (lo, hi)
+// and the plan bounds keys-per-CTA * max|digit| * max|V| by 2^24, so both
+// FP32 accumulators O_lo, O_hi are exact; O = O_lo + (O_hi << shift) in
+// wrapping int32.
 //
 // FP32 kind (3xTF32, kind::tf32): every operand is split into TF32 big +
 // small parts; S_b = Q_big [K_big; K_small]^T + Q_small K_big^T and
@@ -35,33 +38,83 @@
 namespace qx {
 
 namespace attn {
-constexpr int kThreads = 160;       // warps 0-3: S conversion and epilogue; warp 4: TMA + MMA
-constexpr int kConv = 128;          // one converter thread per query row
 constexpr int kQTile = 128;         // queries per CTA
 constexpr int kTmemCols = 512;
-constexpr int kTmemS = 0;           // S block
-constexpr int kTmemO = 256;         // O^T: 256 columns (two halves of 128 queries)
 constexpr int kMaxCluster = 8;
 
-// Integer kind
-constexpr int kKeys = 64;
-constexpr uint32_t kIdescS = make_idesc(128, kKeys, 0);
-constexpr uint32_t kIdescO = make_idesc(128, 256, 0);
+// ---------------------------------------------------------- integer kind
+// Warps 0-7 turn S into FP16 digits in place in TMEM and finally write the
+// partial O; warp 8 issues the TMA loads; warp 9 owns TMEM and issues the
+// MMAs.  A key block holds 128 keys: S_b = Q K_b^T is one N = 128 product
+// per 16 head dimensions, and O += S_b V_b takes its A operand (the digits)
+// straight from TMEM, so the digits never touch shared memory.  S has three
+// TMEM buffers for head sizes up to 64 (two for 128), so the digits of
+// block b+1 are made while the tensor cores run O += S_b V_b and S_{b+2}.
+constexpr int kThreads = 320;
+constexpr int kConv = 256;
+constexpr int kProducerWarp = 8;
+constexpr int kIssuerWarp = 9;
+constexpr int kBlockKeys = 128;                         // keys per S block
+constexpr int kMaxStages = 8;                           // K / V^T ring
+constexpr int kMaxSBufs = 3;
+constexpr uint32_t kIdescS = make_idesc(128, kBlockKeys, 0);
 struct Smem {
     static constexpr int Q_BLK = kQTile * 128;          // one 64-wide k-block of Q
-    static constexpr int K_BLK = kKeys * 128;           // one 64-wide k-block of K
-    static constexpr int VT = 128 * 128;                // 128 rows of V^T x 64 keys
-    static constexpr int S = 256 * 128;                 // both digit tiles
-    static constexpr int KV_STAGE = 2 * K_BLK + VT;     // K (up to 2 k-blocks) + V^T
+    static constexpr int K_BLK = kBlockKeys * 128;      // one 64-wide k-block of 128 keys
     static constexpr int q_off = 0;                     // Q: up to 2 k-blocks
     static constexpr int kv_off = 2 * Q_BLK;
-    static constexpr int s_off = kv_off + 2 * KV_STAGE;
-    static constexpr int part_off = s_off + S;          // partial O: 128 x (64 or 128) int32
-    static constexpr int bar_off = part_off + kQTile * 128 * 4;
+    // Ring stage: dkb k-blocks of K plus V^T as two 64-key halves of dp rows:
+    // 32 KB for dp = 64 (6 stages), 64 KB for dp = 128 (3 stages).
+    static constexpr int RING = 192 * 1024;
+    static constexpr int part_off = kv_off;             // partial O, once the ring is idle
+    static constexpr int bar_off = kv_off + RING;
     static constexpr int total = bar_off + 256 + 1024;
 };
+// row pitch of the partial O in int32 words (conflict-free 16-byte row stores)
+__host__ __device__ constexpr int part_pitch(int pd) { return pd + 4; }
+static_assert(kQTile * part_pitch(128) * 4 <= Smem::RING, "partial O must fit the ring");
+static_assert(Smem::RING / (Smem::K_BLK + 2 * 64 * 128) <= kMaxStages, "ring barriers");
+static_assert(Smem::total <= 227 * 1024, "shared memory");
 
-// FP32 kind
+struct BarsI {
+    uint64_t *q, *kv_full, *kv_empty, *s_full, *sready, *o_done, *tail;
+    uint32_t *tmem_slot;
+    volatile int *abort_flag;
+    __device__ BarsI(uint8_t *base) {
+        uint64_t *b = reinterpret_cast<uint64_t *>(base);
+        q = b;
+        kv_full = b + 1;                     // [kMaxStages]
+        kv_empty = kv_full + kMaxStages;     // [kMaxStages]
+        s_full = kv_empty + kMaxStages;      // [kMaxSBufs]
+        sready = s_full + kMaxSBufs;         // [kMaxSBufs]
+        o_done = sready + kMaxSBufs;         // [kMaxSBufs]
+        tail = o_done + kMaxSBufs;
+        tmem_slot = reinterpret_cast<uint32_t *>(tail + 1);
+        abort_flag = reinterpret_cast<volatile int *>(tail + 2);
+    }
+    __device__ void init() {
+        mbar_init(q, 1);
+        for (int i = 0; i < kMaxStages; ++i) {
+            mbar_init(&kv_full[i], 1);
+            mbar_init(&kv_empty[i], 1);
+        }
+        for (int i = 0; i < kMaxSBufs; ++i) {
+            mbar_init(&s_full[i], 1);
+            mbar_init(&sready[i], kConv / 32);     // one arrival per converter warp
+            mbar_init(&o_done[i], 1);
+        }
+        mbar_init(tail, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+};
+static_assert(1 + 2 * kMaxStages + 3 * kMaxSBufs + 1 + 2 <= 256 / 8, "barrier block");
+
+// ------------------------------------------------------------- FP32 kind
+constexpr int kTmemS = 0;                               // S block
+constexpr int kTmemO = 256;                             // O^T: two halves of 128 queries
+constexpr int kThreads32 = 160;     // warps 0-3: S conversion and epilogue; warp 4: TMA + MMA
+constexpr int kConv32 = 128;
 constexpr int kKeys32 = 32;
 constexpr int kDp32 = 64;                               // head size padded to 64
 constexpr uint32_t kIdescS32 = make_idesc(128, 2 * kKeys32, 2);
@@ -103,7 +156,7 @@ struct Bars {
         mbar_init(&kv[0], 1);
         mbar_init(&kv[1], 1);
         mbar_init(s, 1);
-        mbar_init(sready, kConv);
+        mbar_init(sready, kConv32 / 32);   // one arrival per converter warp
         mbar_init(o, 1);
         mbar_init(tail, 1);
         *abort_flag = 0;
@@ -123,36 +176,78 @@ __device__ __forceinline__ void drain_after_abort(const Bars &b, int issued_kv) 
 }
 
 // Cluster reduction: CTA `rank` adds its slice of the 128 query rows over all
-// `cs` CTAs (rank order) and writes O rows qt*128 + j.  part is [128][pd].
+// `cs` CTAs (rank order) and writes O rows qt*128 + j of head `hd`.  part is
+// [128][pitch] (int32 or float words, pitch a multiple of 4).  Rows of O are
+// written four columns at a time when d is a multiple of 4.
 template <bool FLOAT>
-__device__ __forceinline__ void cluster_reduce_store(const void *part, int pd, int cs, int qt,
+__device__ __forceinline__ void cluster_reduce_store(const void *part, int pitch, int cs, int qt, int hd,
                                                      const AttnArgs &a) {
     const uint32_t rank = cluster_rank();
     const int rows = (kQTile + cs - 1) / cs;
     const int j0 = int(rank) * rows;
-    const int j1 = min(kQTile, j0 + rows);
+    const int j1 = min(min(kQTile, j0 + rows), a.L - qt * kQTile);
+    if (j1 <= j0) return;
+    uint32_t peer[kMaxCluster];                          // part in every CTA of the cluster
     const uint32_t pbase = smem_addr(part);
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r) peer[r] = r < cs ? cluster_map(pbase, uint32_t(r)) : 0u;
+    const int64_t obase = (int64_t(hd) * a.L + int64_t(qt) * kQTile) * a.d;
+    if ((a.d & 3) == 0) {
+        const int groups = a.d >> 2;
+        for (int idx = threadIdx.x; idx < (j1 - j0) * groups; idx += blockDim.x) {
+            const int j = j0 + idx / groups;
+            const int c = 4 * (idx - (idx / groups) * groups);
+            const uint32_t off = uint32_t(j * pitch + c) * 4u;
+            uint4 acc = ld_cluster_v4(peer[0] + off);
+#pragma unroll
+            for (int r = 1; r < kMaxCluster; ++r) {
+                if (r < cs) {
+                    const uint4 v = ld_cluster_v4(peer[r] + off);
+                    if constexpr (FLOAT) {
+                        acc.x = __float_as_uint(__uint_as_float(acc.x) + __uint_as_float(v.x));
+                        acc.y = __float_as_uint(__uint_as_float(acc.y) + __uint_as_float(v.y));
+                        acc.z = __float_as_uint(__uint_as_float(acc.z) + __uint_as_float(v.z));
+                        acc.w = __float_as_uint(__uint_as_float(acc.w) + __uint_as_float(v.w));
+                    } else {
+                        acc.x += v.x;
+                        acc.y += v.y;
+                        acc.z += v.z;
+                        acc.w += v.w;
+                    }
+                }
+            }
+            *reinterpret_cast<uint4 *>(static_cast<uint32_t *>(a.out) + obase + int64_t(j) * a.d + c) = acc;
+        }
+        return;
+    }
     for (int idx = threadIdx.x; idx < (j1 - j0) * a.d; idx += blockDim.x) {
         const int j = j0 + idx / a.d;
         const int c = idx - (idx / a.d) * a.d;
-        const int q = qt * kQTile + j;
-        if (q >= a.L) continue;
-        const uint32_t off = uint32_t(j * pd + c) * 4u;
-        if constexpr (FLOAT) {
-            float acc = 0.f;
-            for (int src = 0; src < cs; ++src)
-                acc += __uint_as_float(ld_cluster_u32(cluster_map(pbase + off, uint32_t(src))));
-            static_cast<float *>(a.out)[int64_t(q) * a.d + c] = acc;
-        } else {
-            uint32_t acc = 0u;
-            for (int src = 0; src < cs; ++src) acc += ld_cluster_u32(cluster_map(pbase + off, uint32_t(src)));
-            static_cast<int32_t *>(a.out)[int64_t(q) * a.d + c] = int32_t(acc);
+        const uint32_t off = uint32_t(j * pitch + c) * 4u;
+        uint32_t acc = ld_cluster_u32(peer[0] + off);
+#pragma unroll
+        for (int r = 1; r < kMaxCluster; ++r) {
+            if (r < cs) {
+                const uint32_t v = ld_cluster_u32(peer[r] + off);
+                if constexpr (FLOAT) acc = __float_as_uint(__uint_as_float(acc) + __uint_as_float(v));
+                else acc += v;
+            }
         }
+        static_cast<uint32_t *>(a.out)[obase + int64_t(j) * a.d + c] = acc;
     }
 }
 }  // namespace attn
 
 // ==================================================================== integer
+// Per key block b (128 keys), S buffer i = b mod nsb, ring stage b mod nst:
+//   issuer      S_i = Q K_b^T                        (M 128 queries, N 128 keys)
+//   converters  S_i -> FP16 digits lo, hi, in place  (keys past the CTA's run -> 0)
+//   issuer      O_lo += lo V_b, O_hi += hi V_b       (A from TMEM, M 128 queries,
+//               N = dp, K 16 keys per step; V_b from the packed V^T)
+// TMEM columns: S_i at 128 i; O_lo at 128 nsb, O_hi right after it (dp each).
+// In S_i the digits of keys 32 g .. 32 g + 31 of half h (64 h + 32 g ..) sit in
+// the 32 columns that held their S values: lo in the first 16 (two keys per
+// column, lower key in the low half), hi in the next 16.
 __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __grid_constant__ AttnArgs a) {
     using namespace attn;
     extern __shared__ uint8_t smem_raw[];
@@ -160,23 +255,28 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sq = smem + Smem::q_off;
     uint8_t *skv = smem + Smem::kv_off;
-    uint8_t *ss = smem + Smem::s_off;
     int32_t *part = reinterpret_cast<int32_t *>(smem + Smem::part_off);
-    Bars bar(smem + Smem::bar_off);
+    BarsI bar(smem + Smem::bar_off);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int cs = a.key_splits;                         // cluster size
     const int qt = blockIdx.x / cs;
     const int split = blockIdx.x - qt * cs;
+    const int hd = blockIdx.y;                           // head
     const int dkb = a.d > 64 ? 2 : 1;                    // 64-wide k-blocks of Q and K
-    const int pd = a.d > 64 ? 128 : 64;                  // row pitch of the partial O
+    const int dp = 64 * dkb;                             // padded head size = N of the O product
+    const int nsb = dkb == 1 ? 3 : 2;                    // S buffers in TMEM
+    const int pitch = part_pitch(dp);
+    const int stage_bytes = dkb * Smem::K_BLK + 2 * dp * 128;
+    const int nst = Smem::RING / stage_bytes;           // 6 or 3 stages
     const int key_begin = split * a.keys_per_split;
-    int nkb = (min(a.L, key_begin + a.keys_per_split) - key_begin + kKeys - 1) / kKeys;
-    if (nkb < 0) nkb = 0;
+    const int key_end = min(a.L, key_begin + a.keys_per_split);
+    int nb = (key_end - key_begin + kBlockKeys - 1) / kBlockKeys;
+    if (nb < 0) nb = 0;
 
     if (threadIdx.x == 0) bar.init();
-    if (warp == 4) {
+    if (warp == kIssuerWarp) {
         tmem_alloc(bar.tmem_slot, kTmemCols);
         tmem_relinquish();
     }
@@ -184,137 +284,220 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *bar.tmem_slot;
-    const uint32_t tS = tmem + kTmemS;
-    const uint32_t tO = tmem + kTmemO;
+    const uint32_t tOlo = tmem + uint32_t(nsb * kBlockKeys);
+    const uint32_t tOhi = tOlo + uint32_t(dp);
     pdl_wait();   // packed operands come from the kernel launched just before
 
     bool ok = true;
-    if (warp == 4) {
-        if (lane == 0 && nkb > 0) {
-            // ------------------------------------------- loads + MMA issue
+    if (warp == kProducerWarp) {
+        // ---------------------------------------------------------- TMA loads
+        if (lane == 0 && nb > 0) {
             tma_prefetch(&a.tm_q);
             tma_prefetch(&a.tm_k);
             tma_prefetch(&a.tm_vt);
             mbar_expect_tx(bar.q, dkb * Smem::Q_BLK);
             for (int kb = 0; kb < dkb; ++kb)
-                tma_load_2d(sq + kb * Smem::Q_BLK, &a.tm_q, bar.q, kb * 64, qt * kQTile);
-            auto load_kv = [&](int b) {
-                uint8_t *st = skv + (b & 1) * Smem::KV_STAGE;
-                const int key0 = key_begin + b * kKeys;
-                mbar_expect_tx(&bar.kv[b & 1], dkb * Smem::K_BLK + Smem::VT);
+                tma_load_3d(sq + kb * Smem::Q_BLK, &a.tm_q, bar.q, kb * 64, qt * kQTile, hd);
+            int issued = 0;
+            for (int b = 0, st = 0, round = 0; b < nb; ++b) {
+                if (round > 0 &&
+                    !mbar_wait(&bar.kv_empty[st], uint32_t((round - 1) & 1), bar.abort_flag, a.err))
+                    break;
+                uint8_t *dst = skv + st * stage_bytes;
+                const int key0 = key_begin + b * kBlockKeys;
+                mbar_expect_tx(&bar.kv_full[st], stage_bytes);
                 for (int kb = 0; kb < dkb; ++kb)
-                    tma_load_2d(st + kb * Smem::K_BLK, &a.tm_k, &bar.kv[b & 1], kb * 64, key0);
-                tma_load_2d(st + 2 * Smem::K_BLK, &a.tm_vt, &bar.kv[b & 1], key0, 0);
-            };
-            load_kv(0);
-            int issued_kv = 1;
-            for (int b = 0; ok && b < nkb; ++b) {
-                if (b + 1 < nkb) {
-                    // stage (b+1)&1 was read by block b-1; its O MMA must be done
-                    if (b >= 1 && !mbar_wait(bar.o, uint32_t((b - 1) & 1), bar.abort_flag, a.err)) {
-                        ok = false;
-                        break;
-                    }
-                    load_kv(b + 1);
-                    ++issued_kv;
+                    tma_load_3d(dst + kb * Smem::K_BLK, &a.tm_k, &bar.kv_full[st], kb * 64, key0, hd);
+                for (int h = 0; h < 2; ++h)
+                    tma_load_3d(dst + dkb * Smem::K_BLK + h * dp * 128, &a.tm_vt, &bar.kv_full[st],
+                                key0 + 64 * h, 0, hd);
+                ++issued;
+                if (++st == nst) {
+                    st = 0;
+                    ++round;
                 }
-                if (b == 0 && !mbar_wait(bar.q, 0, bar.abort_flag, a.err)) {
-                    ok = false;
-                    break;
+            }
+            if (*bar.abort_flag) {
+                // every copy already issued lands before shared memory goes
+                for (int st = 0; st < nst; ++st) {
+                    const int uses = issued / nst + (st < issued % nst ? 1 : 0);
+                    if (uses > 0) mbar_wait_drain(&bar.kv_full[st], uint32_t((uses - 1) & 1));
                 }
-                if (!mbar_wait(&bar.kv[b & 1], uint32_t((b >> 1) & 1), bar.abort_flag, a.err)) {
-                    ok = false;
-                    break;
+                mbar_wait_drain(bar.q, 0);
+            }
+        }
+    } else if (warp == kIssuerWarp) {
+        // ---------------------------------------------------------- MMA issue
+        // The whole warp runs this loop; one elected lane issues each MMA and
+        // commit (warp-uniform operands make the issue cheaper).
+        if (nb > 0) {
+            const uint32_t idesc_o = make_idesc(128, dp, 0);
+            const uint64_t qdesc = make_sdesc(smem_addr(sq));
+            // S runs two key blocks ahead of O; each keeps its own ring position
+            int s_st = 0, s_round = 0, o_st = 0;
+            auto issue_s = [&](int b) -> bool {
+                const int i = b % nsb;
+                // S_i was last read (as digits) by O of block b - nsb
+                if (b >= nsb &&
+                    !mbar_wait_warp(&bar.o_done[i], uint32_t(((b - nsb) / nsb) & 1), bar.abort_flag, a.err))
+                    return false;
+                const int st = s_st;
+                if (!mbar_wait_warp(&bar.kv_full[st], uint32_t(s_round & 1), bar.abort_flag, a.err))
+                    return false;
+                if (++s_st == nst) {
+                    s_st = 0;
+                    ++s_round;
                 }
                 tc_fence_after();
-                const uint32_t qa = smem_addr(sq);
-                const uint32_t ka = smem_addr(skv + (b & 1) * Smem::KV_STAGE);
+                const uint64_t kdesc = make_sdesc(smem_addr(skv + st * stage_bytes));
+                const uint32_t ts = tmem + uint32_t(i * kBlockKeys);
                 for (int kb = 0; kb < dkb; ++kb)
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
-                        mma_f16(tS, make_sdesc(qa + kb * Smem::Q_BLK + kk * 32),
-                                make_sdesc(ka + kb * Smem::K_BLK + kk * 32), kIdescS,
-                                (kb > 0 || kk > 0) ? 1u : 0u);
-                tc_commit(bar.s);
-                if (!mbar_wait(bar.sready, uint32_t(b & 1), bar.abort_flag, a.err)) {
+                        mma_f16_elect(ts, qdesc + uint64_t((kb * Smem::Q_BLK + kk * 32) >> 4),
+                                      kdesc + uint64_t((kb * Smem::K_BLK + kk * 32) >> 4), kIdescS,
+                                      (kb > 0 || kk > 0) ? 1u : 0u);
+                tc_commit_elect(&bar.s_full[i]);
+                return true;
+            };
+            ok = mbar_wait_warp(bar.q, 0, bar.abort_flag, a.err) && issue_s(0) && (nb < 2 || issue_s(1));
+            for (int b = 0; ok && b < nb; ++b) {
+                const int i = b % nsb;
+                const int st = o_st;
+                if (++o_st == nst) o_st = 0;
+                if (!mbar_wait_warp(&bar.sready[i], uint32_t((b / nsb) & 1), bar.abort_flag, a.err)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t va = ka + 2 * Smem::K_BLK;
-                const uint32_t sa = smem_addr(ss);
+                const uint64_t vdesc = make_sdesc(smem_addr(skv + st * stage_bytes + dkb * Smem::K_BLK));
+                const uint32_t ts = tmem + uint32_t(i * kBlockKeys);
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk)
-                    mma_f16(tO, make_sdesc(va + kk * 32), make_sdesc(sa + kk * 32), kIdescO,
-                            (b > 0 || kk > 0) ? 1u : 0u);
-                tc_commit(bar.o);
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const uint64_t vd = vdesc + uint64_t((h * dp * 128 + kk * 32) >> 4);
+                        const uint32_t col = uint32_t(64 * h + 32 * (kk >> 1) + 8 * (kk & 1));
+                        const uint32_t acc = (b > 0 || h > 0 || kk > 0) ? 1u : 0u;
+                        mma_f16_ts_elect(tOlo, ts + col, vd, idesc_o, acc);
+                        mma_f16_ts_elect(tOhi, ts + col + 16u, vd, idesc_o, acc);
+                    }
+                tc_commit_elect(&bar.o_done[i]);
+                tc_commit_elect(&bar.kv_empty[st]);
+                if (b + 2 < nb && !issue_s(b + 2)) ok = false;
             }
-            if (!ok) drain_after_abort(bar, issued_kv);
+            if (!ok) {
+                // MMAs already issued finish before TMEM and shared memory go
+                tc_commit_elect(bar.tail);
+                mbar_wait_drain(bar.tail, 0);
+            }
         }
     } else {
-        // ------------------------------------------- S -> FP16 digits in smem
-        const int row = warp * 32 + lane;                // query row of this thread
-        const int half = 1 << (a.s_shift - 1);
-        const int mask = (1 << a.s_shift) - 1;
-        for (int b = 0; b < nkb; ++b) {
-            if (!mbar_wait(bar.s, uint32_t(b & 1), bar.abort_flag, a.err)) {
-                ok = false;
-                break;
-            }
-            if (b >= 1 && !mbar_wait(bar.o, uint32_t((b - 1) & 1), bar.abort_flag, a.err)) {
+        // -------------------------------------- S -> FP16 digits, in TMEM
+        const int quarter = warp & 3;                    // TMEM lanes 32 quarter ..
+        const int h = warp >> 2;                         // keys 64 h .. 64 h + 63 of a block
+        const int row = quarter * 32 + lane;             // query row of this thread
+        const uint32_t lane_off = uint32_t(quarter * 32) << 16;
+        // Digits of S in the float domain (FMA pipe only; the conversion
+        // unit is far slower): hi = floor(S 2^-s + 1/2), lo = S - hi 2^s,
+        // the same balanced digits as ((S + 2^(s-1)) & (2^s - 1)) - 2^(s-1).
+        // Every step is exact: S is an integer below 2^24 in magnitude, the
+        // FMA adds 1/2 to a power-of-two scaling of it, and |S 2^-s| < 2^22
+        // lets the add of 1.5 * 2^23 rounded down land on floor() exactly.
+        const float inv_scale = __int_as_float((127 - a.s_shift) << 23);   // 2^-s
+        const float scale = __int_as_float((127 + a.s_shift) << 23);       // 2^s
+        constexpr float kMagic = 12582912.0f;                              // 1.5 * 2^23
+        for (int b = 0; b < nb; ++b) {
+            const int i = b % nsb;
+            if (!mbar_wait(&bar.s_full[i], uint32_t((b / nsb) & 1), bar.abort_flag, a.err)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
-            uint8_t *rlo = ss + row * 128;
-            uint8_t *rhi = ss + (128 + row) * 128;
+            const int key0 = key_begin + b * kBlockKeys + 64 * h;
 #pragma unroll
-            for (int p = 0; p < kKeys / 32; ++p) {
+            for (int g = 0; g < 2; ++g) {
+                const uint32_t taddr = tmem + lane_off + uint32_t(i * kBlockKeys + 64 * h + 32 * g);
                 uint32_t v[32];
-                tmem_ld32(tS + (uint32_t(warp * 32) << 16) + p * 32, v);
+                tmem_ld32(taddr, v);
                 tmem_wait_ld(v);
+                const int valid = key_end - (key0 + 32 * g);     // keys of this group in the run
+                if (valid < 32) {                                // past the run: digits 0
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    __align__(16) __half lo[8], hi[8];
+                    for (int x = 0; x < 32; ++x)
+                        if (x >= valid) v[x] = 0u;
+                }
+                uint32_t lo[16], hi[16];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const int32_t sv = __float2int_rn(__uint_as_float(v[c * 8 + e]));
-                        const int32_t d0 = ((sv + half) & mask) - half;
-                        lo[e] = __int2half_rn(d0);
-                        hi[e] = __int2half_rn((sv - d0) >> a.s_shift);
+                for (int e = 0; e < 16; ++e) {
+                    float hv[2], lv[2];
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        const float sv = __uint_as_float(v[2 * e + u]);
+                        hv[u] = __fsub_rn(__fadd_rd(fmaf(sv, inv_scale, 0.5f), kMagic), kMagic);
+                        lv[u] = fmaf(-hv[u], scale, sv);
                     }
-                    const int chunk = p * 4 + c;                     // 16-byte chunk of the row
-                    const int pos = (chunk ^ (row & 7)) << 4;        // 128B swizzle
-                    *reinterpret_cast<uint4 *>(rlo + pos) = *reinterpret_cast<uint4 *>(lo);
-                    *reinterpret_cast<uint4 *>(rhi + pos) = *reinterpret_cast<uint4 *>(hi);
+                    const __half2 l2 = __floats2half2_rn(lv[0], lv[1]);
+                    const __half2 h2 = __floats2half2_rn(hv[0], hv[1]);
+                    lo[e] = *reinterpret_cast<const uint32_t *>(&l2);
+                    hi[e] = *reinterpret_cast<const uint32_t *>(&h2);
                 }
+                tmem_st16(taddr, lo);
+                tmem_st16(taddr + 16u, hi);
             }
-            // generic-proxy smem writes -> visible to the tensor core's async proxy
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            // every lane's TMEM stores are done before lane 0 signals the warp
+            tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(bar.sready);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bar.sready[i]);
         }
-        // ------------------------------- this CTA's partial O -> shared memory
-        const int c = warp * 32 + lane;                  // output column (row of V^T)
-        const bool have = ok && nkb > 0 && mbar_wait(bar.o, uint32_t((nkb - 1) & 1), bar.abort_flag, a.err);
+        // ------------------------ this CTA's partial O -> shared memory
+        // (the K / V^T ring is idle once the last O product has completed)
+        const int last = nb - 1;
+        const bool have = ok && nb > 0 &&
+                          mbar_wait(&bar.o_done[last % nsb], uint32_t((last / nsb) & 1), bar.abort_flag, a.err);
         if (have) tc_fence_after();
-        if (warp * 32 < a.d) {
+        // One CTA per query tile: O rows go straight to global memory.
+        // Otherwise the partial waits in shared memory for the cluster sum.
+        const int q = qt * kQTile + row;
+        int32_t *orow = static_cast<int32_t *>(a.out) + (int64_t(hd) * a.L + q) * a.d;
+        const bool vec = (a.d & 3) == 0;
+        const int cols = dp / 2;                         // output columns of this warp
 #pragma unroll 1
-            for (int p = 0; p < kQTile / 32; ++p) {
-                uint32_t lo[32], hi[32];
-                if (have) {
-                    tmem_ld32(tO + (uint32_t(warp * 32) << 16) + p * 32, lo);
-                    tmem_wait_ld(lo);
-                    tmem_ld32(tO + (uint32_t(warp * 32) << 16) + 128 + p * 32, hi);
-                    tmem_wait_ld(hi);
-                }
+        for (int c0 = h * cols; c0 < (h + 1) * cols; c0 += 32) {
+            uint32_t lo[32], hi[32];
+            if (have) {
+                tmem_ld32(tOlo + lane_off + uint32_t(c0), lo);
+                tmem_ld32(tOhi + lane_off + uint32_t(c0), hi);
+                tmem_wait_ld(lo);
+                tmem_wait_ld(hi);
+            }
+            int32_t *dst = part + row * pitch + c0;
 #pragma unroll
-                for (int x = 0; x < 32; ++x) {
-                    const uint32_t val =
-                        have ? uint32_t(__float2int_rn(__uint_as_float(lo[x]))) +
-                                   (uint32_t(__float2int_rn(__uint_as_float(hi[x]))) << a.s_shift)
-                             : 0u;
-                    if (c < a.d) part[(p * 32 + x) * pd + c] = int32_t(val);
+            for (int x = 0; x < 32; x += 4) {
+                uint4 w = make_uint4(0u, 0u, 0u, 0u);
+                if (have) {
+                    w.x = uint32_t(__float2int_rn(__uint_as_float(lo[x]))) +
+                          (uint32_t(__float2int_rn(__uint_as_float(hi[x]))) << a.s_shift);
+                    w.y = uint32_t(__float2int_rn(__uint_as_float(lo[x + 1]))) +
+                          (uint32_t(__float2int_rn(__uint_as_float(hi[x + 1]))) << a.s_shift);
+                    w.z = uint32_t(__float2int_rn(__uint_as_float(lo[x + 2]))) +
+                          (uint32_t(__float2int_rn(__uint_as_float(hi[x + 2]))) << a.s_shift);
+                    w.w = uint32_t(__float2int_rn(__uint_as_float(lo[x + 3]))) +
+                          (uint32_t(__float2int_rn(__uint_as_float(hi[x + 3]))) << a.s_shift);
+                }
+                if (cs > 1) {
+                    *reinterpret_cast<uint4 *>(dst + x) = w;
+                } else if (q < a.L) {
+                    const int c = c0 + x;
+                    if (vec && c + 3 < a.d) {
+                        *reinterpret_cast<uint4 *>(orow + c) = w;
+                    } else {
+                        if (c < a.d) orow[c] = int32_t(w.x);
+                        if (c + 1 < a.d) orow[c + 1] = int32_t(w.y);
+                        if (c + 2 < a.d) orow[c + 2] = int32_t(w.z);
+                        if (c + 3 < a.d) orow[c + 3] = int32_t(w.w);
+                    }
                 }
             }
         }
@@ -322,17 +505,19 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
 
     tc_fence_before();
     __syncthreads();
-    cluster_sync();                                      // every partial is in place
-    cluster_reduce_store<false>(part, pd, cs, qt, a);
-    cluster_sync();                                      // peers are done reading
-    if (warp == 4) {
+    if (cs > 1) {
+        cluster_sync();                                  // every partial is in place
+        cluster_reduce_store<false>(part, pitch, cs, qt, hd, a);
+        cluster_sync();                                  // peers are done reading
+    }
+    if (warp == kIssuerWarp) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
     }
 }
 
 // ======================================================================= FP32
-__global__ void __launch_bounds__(attn::kThreads, 1)
+__global__ void __launch_bounds__(attn::kThreads32, 1)
     attn_core_f32_kernel(const __grid_constant__ AttnArgs a) {
     using namespace attn;
     extern __shared__ uint8_t smem_raw[];
@@ -349,6 +534,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
     const int cs = a.key_splits;
     const int qt = blockIdx.x / cs;
     const int split = blockIdx.x - qt * cs;
+    const int hd = blockIdx.y;                           // head
     const int key_begin = split * a.keys_per_split;
     int nkb = (min(a.L, key_begin + a.keys_per_split) - key_begin + kKeys32 - 1) / kKeys32;
     if (nkb < 0) nkb = 0;
@@ -374,14 +560,14 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
             tma_prefetch(&a.tm_vt);
             mbar_expect_tx(bar.q, 2 * Smem32::Q_KQ);
             for (int kq = 0; kq < 2; ++kq)
-                tma_load_3d(sq + kq * Smem32::Q_KQ, &a.tm_q, bar.q, kq * 32, qt * kQTile, 0);
+                tma_load_3d(sq + kq * Smem32::Q_KQ, &a.tm_q, bar.q, kq * 32, qt * kQTile, 2 * hd);
             auto load_kv = [&](int b) {
                 uint8_t *st = skv + (b & 1) * Smem32::KV_STAGE;
                 const int key0 = key_begin + b * kKeys32;
                 mbar_expect_tx(&bar.kv[b & 1], Smem32::KV_STAGE);
                 for (int kq = 0; kq < 2; ++kq)
-                    tma_load_3d(st + kq * Smem32::K_KQ, &a.tm_k, &bar.kv[b & 1], kq * 32, key0, 0);
-                tma_load_3d(st + 2 * Smem32::K_KQ, &a.tm_vt, &bar.kv[b & 1], key0, 0, 0);
+                    tma_load_3d(st + kq * Smem32::K_KQ, &a.tm_k, &bar.kv[b & 1], kq * 32, key0, 2 * hd);
+                tma_load_3d(st + 2 * Smem32::K_KQ, &a.tm_vt, &bar.kv[b & 1], key0, 0, 2 * hd);
             };
             load_kv(0);
             int issued_kv = 1;
@@ -464,7 +650,8 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
             }
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             tc_fence_before();
-            mbar_arrive(bar.sready);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar.sready);
         }
         // ------------------------------- this CTA's partial O -> shared memory
         // (the S tile is free once the last O MMA has completed)
@@ -481,19 +668,32 @@ __global__ void __launch_bounds__(attn::kThreads, 1)
                     tmem_wait_ld(lo);
                     tmem_wait_ld(hi);
                 }
+                if (cs > 1) {
 #pragma unroll
-                for (int x = 0; x < 32; ++x)
-                    part[(p * 32 + x) * kDp32 + c] =
-                        have ? __uint_as_float(lo[x]) + __uint_as_float(hi[x]) : 0.f;
+                    for (int x = 0; x < 32; ++x)
+                        part[(p * 32 + x) * kDp32 + c] =
+                            have ? __uint_as_float(lo[x]) + __uint_as_float(hi[x]) : 0.f;
+                } else if (c < a.d) {
+                    // one CTA per query tile: lanes hold consecutive columns of O
+                    float *out = static_cast<float *>(a.out) + int64_t(hd) * a.L * a.d;
+#pragma unroll
+                    for (int x = 0; x < 32; ++x) {
+                        const int q = qt * kQTile + p * 32 + x;
+                        if (q < a.L)
+                            out[int64_t(q) * a.d + c] = have ? __uint_as_float(lo[x]) + __uint_as_float(hi[x]) : 0.f;
+                    }
+                }
             }
         }
     }
 
     tc_fence_before();
     __syncthreads();
-    cluster_sync();
-    cluster_reduce_store<true>(part, kDp32, cs, qt, a);
-    cluster_sync();
+    if (cs > 1) {
+        cluster_sync();
+        cluster_reduce_store<true>(part, kDp32, cs, qt, hd, a);
+        cluster_sync();
+    }
     if (warp == 4) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
@@ -507,8 +707,8 @@ cudaError_t attn_prepare() {
 }
 
 cudaError_t attn_launch(const AttnArgs &a, cudaStream_t stream) {
-    return launch_pdl(attn_core_kernel, a.q_tiles * a.key_splits, attn::kThreads, attn::Smem::total,
-                      stream, a, a.key_splits);
+    return launch_pdl(attn_core_kernel, dim3(a.q_tiles * a.key_splits, a.heads), attn::kThreads,
+                      attn::Smem::total, stream, a, a.key_splits);
 }
 
 cudaError_t attn_f32_prepare() {
@@ -517,7 +717,7 @@ cudaError_t attn_f32_prepare() {
 }
 
 cudaError_t attn_f32_launch(const AttnArgs &a, cudaStream_t stream) {
-    return launch_pdl(attn_core_f32_kernel, a.q_tiles * a.key_splits, attn::kThreads,
+    return launch_pdl(attn_core_f32_kernel, dim3(a.q_tiles * a.key_splits, a.heads), attn::kThreads32,
                       attn::Smem32::total, stream, a, a.key_splits);
 }
 

@@ -68,12 +68,14 @@ struct MmaArgs {
 
 // Kernel arguments of the fused attention core.
 struct AttnArgs {
-    CUtensorMap tm_q;         // Q   (L x d): fp16 2-D, or fp32 3-D (d, L, big/small)
-    CUtensorMap tm_k;         // K   (L x d): same
-    CUtensorMap tm_vt;        // V^T (d x L): fp16 2-D, or fp32 3-D (L, d, big/small)
-    void *out;                // O (L x d): int32 or float
+    CUtensorMap tm_q;         // Q   (heads x L x d): fp16 3-D (d, L, head), or fp32
+                              //     3-D (d, L, 2 head + big/small)
+    CUtensorMap tm_k;         // K   (heads x L x d): same
+    CUtensorMap tm_vt;        // V^T (heads x d x L): fp16 3-D (L, d, head), or fp32
+                              //     3-D (L, d, 2 head + big/small)
+    void *out;                // O (heads x L x d): int32 or float
     int *err;
-    int L, d;
+    int L, d, heads;
     int q_tiles, key_splits, keys_per_split;   // key_splits = cluster size (<= 8)
     int s_shift;              // digit width of the S limbs (integer kind)
     int o_chunk_kb;           // key-blocks per FP32 chunk of the second product

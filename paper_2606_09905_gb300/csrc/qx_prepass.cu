@@ -300,15 +300,18 @@ __global__ void __launch_bounds__(256) pack_conv_f32_kernel(const ConvPackF32Arg
 }
 
 // ------------------------------------------------------- attention operands
+// Q, K, V are heads x L x d.  Q and K become [head][L][dp] FP16 (one head
+// after another, so the rows are simply the heads * L input rows); V becomes
+// [head][dp][Lp] (transposed per head, keys contiguous).
 struct AttnPackArgs {
     const void *Q, *K, *V;
-    int L, d, dp, Lp;
-    __half *q, *k;          // L x dp each
-    __half *vt;             // dp x Lp (V transposed, keys contiguous)
+    int heads, L, d, dp, Lp;
+    __half *q, *k;          // heads*L x dp each
+    __half *vt;             // heads x dp x Lp
     RangeCheck cq, ck, cv;
     int *err;
     int qk_blocks;          // blocks [0, qk_blocks) pack Q and K; the rest transpose V
-    int v_tiles_l;
+    int v_tiles_l, v_tiles_c;
 };
 
 template <typename T>
@@ -320,13 +323,14 @@ __global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
     const T *V = static_cast<const T *>(p.V);
     if (int(blockIdx.x) < p.qk_blocks) {
         const int gpr = p.dp >> 3;
-        const int64_t items = int64_t(2) * p.L * gpr;
+        const int64_t rows = int64_t(p.heads) * p.L;
+        const int64_t items = 2 * rows * gpr;
         for (int64_t it = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; it < items;
              it += int64_t(p.qk_blocks) * blockDim.x) {
-            const int which = int(it / (int64_t(p.L) * gpr));
-            const int64_t rem = it - int64_t(which) * p.L * gpr;
-            const int row = int(rem / gpr);
-            const int c = int(rem - int64_t(row) * gpr) * 8;
+            const int which = int(it / (rows * gpr));
+            const int64_t rem = it - which * rows * gpr;
+            const int64_t row = rem / gpr;
+            const int c = int(rem - row * gpr) * 8;
             const T *src = (which ? K : Q) + int64_t(row) * p.d;
             const RangeCheck &ch = which ? p.ck : p.cq;
             int32_t v[8];
@@ -342,14 +346,18 @@ __global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
         }
         return;
     }
-    const int t = int(blockIdx.x) - p.qk_blocks;
+    const int per_head = p.v_tiles_l * p.v_tiles_c;
+    const int hd = (int(blockIdx.x) - p.qk_blocks) / per_head;
+    const int t = int(blockIdx.x) - p.qk_blocks - hd * per_head;
     const int l0 = (t % p.v_tiles_l) * 64;
     const int c0 = (t / p.v_tiles_l) * 64;
+    const T *Vh = V + int64_t(hd) * p.L * p.d;
+    __half *vth = p.vt + int64_t(hd) * p.dp * p.Lp;
     for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
         const int lr = i >> 6, cc = i & 63;
         int32_t v = 0;
         if (l0 + lr < p.L && c0 + cc < p.d) {
-            v = int32_t(V[int64_t(l0 + lr) * p.d + c0 + cc]);
+            v = int32_t(Vh[int64_t(l0 + lr) * p.d + c0 + cc]);
             p.cv.test(v, p.err);
         }
         tile[lr][cc] = v;
@@ -362,16 +370,16 @@ __global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
         int32_t v[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) v[e] = tile[lg * 8 + e][cr];
-        store_limbs8<1>(p.vt + int64_t(c) * p.Lp + l, 0, v, 0);
+        store_limbs8<1>(vth + int64_t(c) * p.Lp + l, 0, v, 0);
     }
 }
 
 // ------------------------------------------------ attention, FP32 kind
-// Q, K (L x d) -> big/small TF32 planes [2][L][64] (zero columns beyond d);
-// V -> V^T planes [2][64][Lp].
+// Q, K (heads x L x d) -> big/small TF32 planes [head][2][L][64] (zero
+// columns beyond d); V -> V^T planes [head][2][64][Lp].
 struct AttnPackF32Args {
     const float *Q, *K, *V;
-    int L, d, Lp;
+    int heads, L, d, Lp;
     float *q, *k, *vt;
     int qk_blocks, v_tiles_l;
 };
@@ -380,26 +388,31 @@ __global__ void __launch_bounds__(256) pack_attn_f32_kernel(const AttnPackF32Arg
     pdl_launch_dependents();
     __shared__ float tile[64][65];
     if (int(blockIdx.x) < p.qk_blocks) {
-        const int64_t items = int64_t(2) * p.L * 8;            // 8 groups of 8 columns
+        const int64_t rows = int64_t(p.heads) * p.L;
+        const int64_t items = 2 * rows * 8;                    // 8 groups of 8 columns
         for (int64_t it = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; it < items;
              it += int64_t(p.qk_blocks) * blockDim.x) {
-            const int which = int(it / (int64_t(p.L) * 8));
-            const int64_t rem = it - int64_t(which) * p.L * 8;
-            const int row = int(rem / 8);
+            const int which = int(it / (rows * 8));
+            const int64_t rem = it - which * rows * 8;
+            const int64_t row = rem / 8;
             const int c = int(rem % 8) * 8;
-            const float *src = (which ? p.K : p.Q) + int64_t(row) * p.d;
+            const int64_t hd = row / p.L;
+            const float *src = (which ? p.K : p.Q) + row * p.d;
             float v[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e) v[e] = c + e < p.d ? src[c + e] : 0.f;
-            store_split8((which ? p.k : p.q) + int64_t(row) * 64 + c, int64_t(p.L) * 64, v);
+            // row l of head hd sits at (2 hd) L + l: the big plane of that head
+            store_split8((which ? p.k : p.q) + (row + hd * p.L) * 64 + c, int64_t(p.L) * 64, v);
         }
         return;
     }
-    const int t = int(blockIdx.x) - p.qk_blocks;
-    const int l0 = t * 64;
+    const int hd = (int(blockIdx.x) - p.qk_blocks) / p.v_tiles_l;
+    const int l0 = (int(blockIdx.x) - p.qk_blocks - hd * p.v_tiles_l) * 64;
+    const float *Vh = p.V + int64_t(hd) * p.L * p.d;
+    float *vth = p.vt + int64_t(hd) * 2 * 64 * p.Lp;
     for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
         const int lr = i >> 6, cc = i & 63;
-        tile[lr][cc] = (l0 + lr < p.L && cc < p.d) ? p.V[int64_t(l0 + lr) * p.d + cc] : 0.f;
+        tile[lr][cc] = (l0 + lr < p.L && cc < p.d) ? Vh[int64_t(l0 + lr) * p.d + cc] : 0.f;
     }
     __syncthreads();
     for (int i = threadIdx.x; i < 64 * 8; i += blockDim.x) {
@@ -409,7 +422,7 @@ __global__ void __launch_bounds__(256) pack_attn_f32_kernel(const AttnPackF32Arg
         float v[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) v[e] = tile[lg * 8 + e][cr];
-        store_split8(p.vt + int64_t(cr) * p.Lp + l, int64_t(64) * p.Lp, v);
+        store_split8(vth + int64_t(cr) * p.Lp + l, int64_t(64) * p.Lp, v);
     }
 }
 
@@ -536,14 +549,15 @@ cudaError_t launch_pack_conv_f32(const float *x, const float *w, int n, int c, i
     return cudaGetLastError();
 }
 
-cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int L, int d,
-                             int dp, int Lp, __half *q, __half *k, __half *vt, int check,
+cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int heads, int L,
+                             int d, int dp, int Lp, __half *q, __half *k, __half *vt, int check,
                              qx_range rq, qx_range rk, qx_range rv, int *err, int num_sms,
                              cudaStream_t st) {
     AttnPackArgs p;
     p.Q = Q;
     p.K = K;
     p.V = V;
+    p.heads = heads;
     p.L = L;
     p.d = d;
     p.dp = dp;
@@ -555,12 +569,14 @@ cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void 
     p.ck = make_check(check, rk);
     p.cv = make_check(check, rv);
     p.err = err;
-    const int64_t qk_items = int64_t(2) * L * (dp / 8);
+    const int64_t qk_items = int64_t(2) * heads * L * (dp / 8);
     int64_t qk_blocks = (qk_items + 255) / 256;
-    if (qk_blocks > num_sms) qk_blocks = num_sms;
+    if (qk_blocks > int64_t(num_sms) * 4) qk_blocks = int64_t(num_sms) * 4;
     p.qk_blocks = int(qk_blocks);
     p.v_tiles_l = (Lp + 63) / 64;
-    const int grid = p.qk_blocks + p.v_tiles_l * ((dp + 63) / 64);
+    p.v_tiles_c = (dp + 63) / 64;
+    const int64_t grid = p.qk_blocks + int64_t(heads) * p.v_tiles_l * p.v_tiles_c;
+    if (grid > INT32_MAX) return cudaErrorInvalidValue;
     if (i32) pack_attn_kernel<int32_t><<<grid, 256, 0, st>>>(p);
     else pack_attn_kernel<int16_t><<<grid, 256, 0, st>>>(p);
     return cudaGetLastError();
@@ -569,24 +585,27 @@ cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void 
 }  // namespace qx
 
 namespace qx {
-cudaError_t launch_pack_attn_f32(const float *Q, const float *K, const float *V, int L, int d, int Lp,
-                                 float *q, float *k, float *vt, int num_sms, cudaStream_t st) {
+cudaError_t launch_pack_attn_f32(const float *Q, const float *K, const float *V, int heads, int L, int d,
+                                 int Lp, float *q, float *k, float *vt, int num_sms, cudaStream_t st) {
     AttnPackF32Args p;
     p.Q = Q;
     p.K = K;
     p.V = V;
+    p.heads = heads;
     p.L = L;
     p.d = d;
     p.Lp = Lp;
     p.q = q;
     p.k = k;
     p.vt = vt;
-    const int64_t items = int64_t(2) * L * 8;
+    const int64_t items = int64_t(2) * heads * L * 8;
     int64_t blocks = (items + 255) / 256;
-    if (blocks > num_sms) blocks = num_sms;
+    if (blocks > int64_t(num_sms) * 4) blocks = int64_t(num_sms) * 4;
     p.qk_blocks = int(blocks < 1 ? 1 : blocks);
     p.v_tiles_l = (Lp + 63) / 64;
-    pack_attn_f32_kernel<<<p.qk_blocks + p.v_tiles_l, 256, 0, st>>>(p);
+    const int64_t grid = p.qk_blocks + int64_t(heads) * p.v_tiles_l;
+    if (grid > INT32_MAX) return cudaErrorInvalidValue;
+    pack_attn_f32_kernel<<<int(grid), 256, 0, st>>>(p);
     return cudaGetLastError();
 }
 }  // namespace qx

@@ -55,15 +55,17 @@ def conv_case_f32(n, c, h, w, k, r, s, seed):
 
 
 def attn_case(L: int, d: int, lo: int, hi: int, seed: int,
-              dtype: torch.dtype = torch.int16):
-    """Q, K, V, each L x d row-major."""
+              dtype: torch.dtype = torch.int16, heads: int = 0):
+    """Q, K, V, each L x d row-major; heads >= 1 gives heads x L x d."""
     g = _gen(seed)
-    return tuple(int_uniform((L, d), lo, hi, g, dtype) for _ in range(3))
+    shape = (L, d) if heads == 0 else (heads, L, d)
+    return tuple(int_uniform(shape, lo, hi, g, dtype) for _ in range(3))
 
 
-def attn_case_f32(L: int, d: int, seed: int):
+def attn_case_f32(L: int, d: int, seed: int, heads: int = 0):
     g = _gen(seed)
-    return tuple(normal((L, d), g) for _ in range(3))
+    shape = (L, d) if heads == 0 else (heads, L, d)
+    return tuple(normal(shape, g) for _ in range(3))
 
 
 @dataclass(frozen=True)

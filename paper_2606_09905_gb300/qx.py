@@ -51,7 +51,7 @@ class PlanDesc(ctypes.Structure):
                 ("s", ctypes.c_int64), ("stride", ctypes.c_int64), ("pad", ctypes.c_int64),
                 ("L", ctypes.c_int64), ("d", ctypes.c_int64),
                 ("range_a", Range), ("range_b", Range), ("range_c", Range),
-                ("flags", ctypes.c_uint)]
+                ("flags", ctypes.c_uint), ("heads", ctypes.c_int64)]
 
 
 class SchemeInfo(ctypes.Structure):
@@ -131,9 +131,9 @@ def conv_desc(n, c, h, w, k_out, r, s, stride, pad, range_x, range_w, dtype=I16,
                     flags=flags)
 
 
-def attn_desc(L, d, range_q, range_k, range_v, dtype=I16, flags=0) -> PlanDesc:
+def attn_desc(L, d, range_q, range_k, range_v, dtype=I16, flags=0, heads=1) -> PlanDesc:
     return PlanDesc(op=OP_ATTN, in_dtype=dtype, L=L, d=d, range_a=_rng(range_q),
-                    range_b=_rng(range_k), range_c=_rng(range_v), flags=flags)
+                    range_b=_rng(range_k), range_c=_rng(range_v), flags=flags, heads=heads)
 
 
 def minmax_desc(count, dtype=I32) -> PlanDesc:
@@ -312,12 +312,15 @@ class Plan:
 
     # -- attention ----------------------------------------------------------
     def attn(self, Q, K, V, O=None, stream=None):
+        """O = (Q K^T) V per head.  Tensors are (L, d) for a single-head plan
+        (or (1, L, d)) and (heads, L, d) otherwise."""
         d = self.desc
         dt = _TORCH_DT[d.in_dtype]
         out_dt = torch.float32 if d.in_dtype == F32 else torch.int32
+        heads = max(1, d.heads)
+        shape = (d.L, d.d) if heads == 1 and Q.dim() == 2 else (heads, d.L, d.d)
         if O is None:
-            O = torch.empty((d.L, d.d), dtype=out_dt, device=Q.device)
-        shape = (d.L, d.d)
+            O = torch.empty(shape, dtype=out_dt, device=Q.device)
         pq, pk, pv = (_ptr(t, dt, shape, n) for t, n in ((Q, "Q"), (K, "K"), (V, "V")))
         po = _ptr(O, out_dt, shape, "O")
         _check(load().qx_attn_core(self.handle, pq, pk, pv, po, _stream(stream)), "qx_attn_core")

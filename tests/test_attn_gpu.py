@@ -77,6 +77,79 @@ def test_attn_identity_reassociation():
     assert_exact(got, q @ (k.T @ v), f"reassociation {info}")
 
 
+# ------------------------------------------------- batched (multi-head) cores
+def attn_gpu_heads(Q, K, V, rq, rk, rv, dtype=qx.I16):
+    H, L, d = Q.shape
+    with qx.Plan(qx.attn_desc(L, d, rq, rk, rv, dtype=dtype, heads=H)) as plan:
+        O = plan.attn(Q.cuda(), K.cuda(), V.cuda())
+        torch.cuda.synchronize()
+        st = plan.status()
+    out = O.cpu().numpy()
+    return (out.astype(np.float64) if dtype == qx.F32 else out.astype(np.int64)), st
+
+
+@pytest.mark.parametrize("H,L,d", [(2, 1024, 64), (5, 100, 64), (3, 129, 8), (12, 300, 128),
+                                   (4, 640, 96), (1, 257, 64), (160, 128, 64)])
+def test_attn_heads_int16(H, L, d):
+    # ragged L and d per head: a tile must never read or write the next head
+    Q, K, V = inputs.attn_case(L, d, -7, 7, seed=H * 1000 + L + d, heads=H)
+    ref, _, _ = oracle.attn(Q, K, V)
+    got, st = attn_gpu_heads(Q, K, V, (-7, 7), (-7, 7), (-7, 7))
+    assert st == qx.OK
+    assert_exact(got, ref, f"attn heads={H} L={L} d={d}")
+
+
+def test_attn_heads_int32_wide():
+    Q, K, V = inputs.attn_case(384, 32, -60, 60, seed=31, dtype=torch.int32, heads=6)
+    ref, _, _ = oracle.attn(Q, K, V)
+    got, st = attn_gpu_heads(Q, K, V, (-60, 60), (-60, 60), (-60, 60), dtype=qx.I32)
+    assert st == qx.OK
+    assert_exact(got, ref, "attn int32 heads=6")
+
+
+def test_attn_heads_zero_means_one():
+    # a descriptor that leaves the head count at 0 is the single-head core
+    Q, K, V = inputs.attn_case(200, 64, -7, 7, seed=32)
+    d = qx.attn_desc(200, 64, (-7, 7), (-7, 7), (-7, 7), heads=0)
+    with qx.Plan(d) as plan:
+        O = plan.attn(Q.cuda(), K.cuda(), V.cuda())
+        O3 = plan.attn(Q.cuda()[None], K.cuda()[None], V.cuda()[None])
+        torch.cuda.synchronize()
+        assert plan.status() == qx.OK
+    ref, _, _ = oracle.attn(Q, K, V)
+    assert_exact(O.cpu().numpy().astype(np.int64), ref, "heads=0")
+    assert_exact(O3.cpu().numpy()[0].astype(np.int64), ref, "heads=0, 3-D tensors")
+
+
+def test_attn_heads_sampled_large():
+    # 32 heads x L = 2048: the full output on the GPU, the oracle on three heads
+    H, L, d = 32, 2048, 64
+    Q, K, V = inputs.attn_case(L, d, -7, 7, seed=33, heads=H)
+    got, st = attn_gpu_heads(Q, K, V, (-7, 7), (-7, 7), (-7, 7))
+    assert st == qx.OK
+    for h in (0, 17, 31):
+        ref, _, _ = oracle.attn(Q[h], K[h], V[h])
+        assert_exact(got[h], ref, f"head {h}")
+
+
+@pytest.mark.parametrize("H,L,d", [(8, 512, 64), (3, 129, 8), (5, 100, 48)])
+def test_attn_heads_f32(H, L, d):
+    Q, K, V = inputs.attn_case_f32(L, d, seed=H * 100 + L + d, heads=H)
+    got, st = attn_gpu_heads(Q, K, V, (0, 0), (0, 0), (0, 0), dtype=qx.F32)
+    assert st == qx.OK
+    within_tolerance(got, Q, K, V, f"attn fp32 heads={H} L={L} d={d}")
+
+
+def test_attn_heads_range_check_flags_a_bad_head():
+    # the device range check covers every head, not just the first
+    Q, K, V = inputs.attn_case(128, 64, -7, 7, seed=34, heads=4)
+    V[3, 127, 63] = 8
+    with qx.Plan(qx.attn_desc(128, 64, (-7, 7), (-7, 7), (-7, 7), heads=4,
+                              flags=qx.FLAG_CHECK_RANGES)) as plan:
+        plan.attn(Q.cuda(), K.cuda(), V.cuda())
+        assert plan.status() == qx.ERR_CONTRACT
+
+
 # ------------------------------------------------------------ FP32 (3xTF32)
 def attn_gpu_f32(Q, K, V):
     L, d = Q.shape

@@ -201,6 +201,32 @@ def test_attn_extremes_and_numpy():
     assert (S == q @ k.T).all() and (O == (q @ k.T) @ v).all()
 
 
+def test_attn_heads_hand_example(golden):
+    g = golden["attn_2heads"]
+    O, S, worst = oracle.attn(np.array(g["Q"]), np.array(g["K"]), np.array(g["V"]))
+    assert O.tolist() == g["O"] and S.shape == (2, 2, 2) and worst == 6
+    assert O[0].tolist() == golden["attn_2x2"]["O"]
+
+
+def test_attn_heads_are_independent():
+    # numpy's batched matmul is the independent routine; permuting the heads
+    # permutes the outputs, and emptying one head's V empties only its output
+    Q, K, V = (t.numpy().astype(np.int64)
+               for t in inputs.attn_case(19, 6, -7, 7, seed=21, heads=3))
+    O, S, worst = oracle.attn(Q, K, V)
+    assert O.shape == (3, 19, 6) and S.shape == (3, 19, 19)
+    assert (S == Q @ K.transpose(0, 2, 1)).all() and (O == (Q @ K.transpose(0, 2, 1)) @ V).all()
+    assert worst == int(np.abs(S).max())
+    perm = [2, 0, 1]
+    assert (oracle.attn(Q[perm], K[perm], V[perm])[0] == O[perm]).all()
+    V0 = V.copy()
+    V0[1] = 0
+    O0 = oracle.attn(Q, K, V0)[0]
+    assert (O0[1] == 0).all() and (O0[0] == O[0]).all() and (O0[2] == O[2]).all()
+    Of, _ = oracle.attn_f64(Q.astype(np.float64), K.astype(np.float64), V.astype(np.float64))
+    assert (Of == O).all()
+
+
 # ----------------------------------------------------------------- FP64 pins
 def test_f64_integer_valued_inputs_are_exact():
     A, B = inputs.gemm_case(20, 30, 40, -1023, 1023, seed=11)
