@@ -266,9 +266,11 @@ def operators(torch, qx, inputs, dev, only=None):
         r["roofline"] = op_roofline(m * conv_ops, tensor_peak, nbytes, peaks["hbm_gbs"], r["execute_ms"])
         return r
 
-    def attn(dtype, H=0, L=1024, d=64):
-        # H = 0: the paper's single-head core; H >= 1: that many independent heads
-        attn_ops = 4.0 * max(1, H) * L * L * d
+    def attn(dtype, H=0, L=1024, d=64, reassoc=False):
+        # H = 0: the paper's single-head core; H >= 1: that many independent heads.
+        # reassoc: O = Q (K^T V), whose own work is 4 L d^2 per head; its rate
+        # on the 4 L^2 d of the order as written is reported beside it.
+        attn_ops = 4.0 * max(1, H) * L * d * (d if reassoc else L)
         if dtype == qx.F32:
             Q, K, V = inputs.attn_case_f32(L, d, seed=0, heads=H)
             rng, desc = (0, 0), "fp32 N(0,1), 3xTF32"
@@ -278,10 +280,14 @@ def operators(torch, qx, inputs, dev, only=None):
             rng, desc = (-7, 7), f"{'int16' if dtype == qx.I16 else 'int32'} in [-7,7]"
         Q, K, V = Q.to(dev), K.to(dev), V.to(dev)
         O = torch.empty(Q.shape, dtype=torch.float32 if dtype == qx.F32 else torch.int32, device=dev)
-        plan_desc = qx.attn_desc(L, d, rng, rng, rng, dtype=dtype, heads=max(1, H))
+        plan_desc = qx.attn_desc(L, d, rng, rng, rng, dtype=dtype, heads=max(1, H),
+                                 flags=qx.FLAG_ATTN_REASSOC if reassoc else 0)
         r = op_times(torch, lambda: qx.Plan(plan_desc), lambda p: p.attn(Q, K, V, O), attn_ops, 50, dev)
         shape = f"{L}x{d}" if H == 0 else f"{H} heads x {L}x{d}"
-        r["workload"] = f"Q,K,V {shape}, O=(QK^T)V, no softmax, {desc}"
+        order = "O=Q(K^T V) (reassociated, same integers)" if reassoc else "O=(QK^T)V"
+        r["workload"] = f"Q,K,V {shape}, {order}, no softmax, {desc}"
+        if reassoc:
+            r["equivalent_gops"] = round(4.0 * max(1, H) * L * L * d / (r["execute_ms"] * 1e-3) / 1e9, 1)
         s0, s1 = qx.query(plan_desc)
         flops = (s0["mma_per_kstep"] + s1["mma_per_kstep"]) * attn_ops / 2.0
         esz = Q.element_size()
@@ -334,7 +340,9 @@ def operators(torch, qx, inputs, dev, only=None):
              "conv_fp32": lambda: conv(qx.F32), "attn_int16": lambda: attn(qx.I16),
              "attn_int32": lambda: attn(qx.I32), "attn_fp32": lambda: attn(qx.F32),
              "attn_mh_int16": lambda: attn(qx.I16, H=32, L=2048),
-             "attn_mh_fp32": lambda: attn(qx.F32, H=32, L=2048)}
+             "attn_mh_fp32": lambda: attn(qx.F32, H=32, L=2048),
+             "attn_ra_int16": lambda: attn(qx.I16, reassoc=True),
+             "attn_mh_ra_int16": lambda: attn(qx.I16, H=32, L=2048, reassoc=True)}
     return {k: f() for k, f in table.items() if only is None or k in only}
 
 

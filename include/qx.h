@@ -80,6 +80,14 @@ typedef struct {
 /* Ask the device to check every operand against its declared range. */
 #define QX_FLAG_CHECK_RANGES 1u
 
+/* Attention plans (integer in_dtype only): compute O = Q (K^T V) instead of
+ * (Q K^T) V.  For integers the two are the same exact result (matrix products
+ * associate in Z and modulo 2^32); the reassociated order does O(L d^2)
+ * instead of O(L^2 d) work and never forms S.  It is a variant of the
+ * Methodology's core, reported on its own.  Extra contract:
+ * L * max|K| * max|V| < 2^31 (the entries of K^T V as int32). */
+#define QX_FLAG_ATTN_REASSOC 2u
+
 typedef struct {
     qx_op op;
     qx_dtype in_dtype; /* I16 or I32 operands -> int32 output; F32 -> float */

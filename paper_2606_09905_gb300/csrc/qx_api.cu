@@ -57,8 +57,10 @@ cudaError_t launch_pack_conv(bool i32, const void *x, const void *w, int n, int 
                              int k_out, int r, int s, int Cp, __half *x_planes, __half *w_planes,
                              int nx, int shift_x, int nw, int shift_w, int check, qx_range rx,
                              qx_range rw, int *err, int num_sms, cudaStream_t st);
+cudaError_t attn_reassoc_prepare();
+cudaError_t attn_reassoc_launch(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int heads, int L, int d,
-                             int dp, int Lp, __half *q, __half *k, __half *vt, int int_check,
+                             int dp, int Lp, __half *q, __half *k, __half *vt, __half *kt, int int_check,
                              qx_range rq, qx_range rk, qx_range rv, int *err, int num_sms,
                              cudaStream_t st);
 
@@ -116,6 +118,7 @@ struct qx_plan_s {
     AttnArgs attn{};
     int s_shift = 0, max_keys = 0, dp = 0, Lp = 0;
     __half *aq = nullptr, *ak = nullptr, *avt = nullptr;
+    __half *akt = nullptr;                                 // K^T, reassociated order
     float *fq = nullptr, *fk = nullptr, *fvt = nullptr;   // FP32 kind
 };
 
@@ -186,6 +189,10 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
         return fail(QX_ERR_UNSUPPORTED, "FP32 plans exist for conv and attention only");
     const bool i16 = d->in_dtype == QX_I16;
     const bool f32 = d->in_dtype == QX_F32;
+    if ((d->flags & QX_FLAG_ATTN_REASSOC) && d->op != QX_OP_ATTN)
+        return fail(QX_ERR_INVALID_ARG, "QX_FLAG_ATTN_REASSOC applies to attention plans only");
+    if ((d->flags & QX_FLAG_ATTN_REASSOC) && f32)
+        return fail(QX_ERR_UNSUPPORTED, "the reassociated attention order is exact for integer plans only");
     auto range_ok = [&](qx_range r) {
         if (f32) return true;   // no range contract for FP32 operands
         if (bad_range(r)) return false;
@@ -269,6 +276,58 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
             const int64_t qm = mag(d->range_a), km = mag(d->range_b), vm = mag(d->range_c);
             if (qm > kHalfExact || km > kHalfExact || vm > kHalfExact)
                 return fail(QX_ERR_CONTRACT, "attention operands must lie within +-2048");
+            if (d->flags & QX_FLAG_ATTN_REASSOC) {
+                // Phase 1: W^T = V^T K, every CTA summing at most kc keys in FP32.
+                const int64_t per = std::max<int64_t>(1, km * vm);
+                const int64_t kc = (kAccLimit / per) / 64 * 64;
+                if (kc < 64) return fail(QX_ERR_CONTRACT, "max|K| * max|V| leaves no exact key chunk");
+                const int64_t chunks = (d->L + kc - 1) / kc;
+                if (chunks > 8)
+                    return fail(QX_ERR_UNSUPPORTED, "L * max|K| * max|V| needs more than 8 exact key chunks");
+                const int64_t wmax = d->L * km * vm;
+                if (wmax > INT32_MAX) return fail(QX_ERR_CONTRACT, "L * max|K| * max|V| exceeds int32");
+                // Phase 2: O = Q W with W in nd balanced digits; d * max|Q| * max|digit| <= 2^24.
+                const int dpad = d->d <= 64 ? 64 : 128;
+                Split best;
+                int64_t best_b = INT64_MAX;
+                for (int nd = 1; nd <= 3 && best_b == INT64_MAX; ++nd) {
+                    if (nd * dpad > 256) break;
+                    for (int sh = 1; sh <= (nd == 1 ? 1 : 12); ++sh) {   // one digit: the shift is unused
+                        Split sp;
+                        if (!make_split(qx_range{-wmax, wmax}, nd, sh, &sp)) continue;
+                        int64_t b = 0;
+                        for (int i = 0; i < nd; ++i) b = std::max(b, sp.bound[i]);
+                        if (d->d * std::max<int64_t>(1, qm) * b > kAccLimit) continue;
+                        if (b < best_b) {
+                            best_b = b;
+                            best = sp;
+                        }
+                    }
+                }
+                if (best_b == INT64_MAX) return fail(QX_ERR_CONTRACT, "no exact digit split of K^T V for Q (K^T V)");
+                Scheme s0, s1;
+                s0.n.limbs = 1;
+                s0.n.bound[0] = km;
+                s0.m.limbs = 1;
+                s0.m.bound[0] = vm;
+                s0.k = d->L;
+                s0.chunk_kb = kc / kBK;
+                s0.n_chunks = chunks;
+                s0.acc_bound = std::min<int64_t>(kc, d->L) * per;
+                s1.n = best;
+                s1.m.limbs = 1;
+                s1.m.bound[0] = qm;
+                s1.k = d->d;
+                s1.chunk_kb = (d->d + kBK - 1) / kBK;
+                s1.n_chunks = 1;
+                s1.acc_bound = d->d * qm * best_b;
+                out[0] = s0;
+                out[1] = s1;
+                *count = 2;
+                if (s_shift) *s_shift = best.shift;
+                if (max_keys) *max_keys = int(std::min<int64_t>(kc, INT32_MAX / 2));
+                return QX_OK;
+            }
             const int64_t smax = d->d * qm * km;
             if (smax > kAccLimit)
                 return fail(QX_ERR_CONTRACT, "d*max|Q|*max|K| exceeds 2^24");
@@ -614,9 +673,73 @@ static qx_status build_attn_f32(qx_plan p) {
     return QX_OK;
 }
 
+// Reassociated order O = Q (K^T V): Q packed by rows, K and V transposed;
+// one cluster per head whose CTAs split the keys (phase 1) and the query
+// rows (phase 2).
+static qx_status build_attn_reassoc(qx_plan p) {
+    const qx_plan_desc &d = p->desc;
+    const uint64_t H = uint64_t(d.heads);
+    p->dp = d.d <= 64 ? 64 : 128;
+    p->Lp = int((d.L + 7) / 8 * 8);
+    const size_t q_bytes = size_t(H) * d.L * p->dp * 2;
+    const size_t t_bytes = size_t(H) * p->dp * p->Lp * 2;
+    p->ws_bytes = 256 + align256(q_bytes) + 2 * align256(t_bytes);
+    QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
+    char *base = static_cast<char *>(p->ws);
+    p->err = reinterpret_cast<int *>(base);
+    p->aq = reinterpret_cast<__half *>(base + 256);
+    p->akt = reinterpret_cast<__half *>(base + 256 + align256(q_bytes));
+    p->avt = reinterpret_cast<__half *>(base + 256 + align256(q_bytes) + align256(t_bytes));
+    QX_CUDA(cudaMemset(p->err, 0, sizeof(int)), "error word reset");
+
+    AttnArgs &a = p->attn;
+    memset(&a, 0, sizeof a);
+    {
+        const uint64_t dims[3] = {uint64_t(p->dp), uint64_t(d.L), H};
+        const uint64_t str[2] = {uint64_t(p->dp) * 2, uint64_t(d.L) * p->dp * 2};
+        const uint32_t box[3] = {64, 128, 1};    // 128 queries
+        qx_status st = encode_tiled(&a.tm_q, p->aq, 3, dims, str, box);
+        if (st != QX_OK) return st;
+    }
+    {
+        const uint64_t dims[3] = {uint64_t(d.L), uint64_t(p->dp), H};
+        const uint64_t str[2] = {uint64_t(p->Lp) * 2, uint64_t(p->dp) * p->Lp * 2};
+        const uint32_t box_v[3] = {64, 128, 1};          // phase 1 A: 128 rows of V^T (zeros past dp)
+        const uint32_t box_k[3] = {64, uint32_t(p->dp), 1};
+        qx_status st = encode_tiled(&a.tm_vt, p->avt, 3, dims, str, box_v);
+        if (st != QX_OK) return st;
+        st = encode_tiled(&a.tm_k, p->akt, 3, dims, str, box_k);
+        if (st != QX_OK) return st;
+    }
+    a.err = p->err;
+    a.L = int(d.L);
+    a.d = int(d.d);
+    a.heads = int(d.heads);
+    a.s_shift = p->scheme[1].n.shift;
+    a.ra_digits = p->scheme[1].n.limbs;
+    a.ra_fast_cvt = p->scheme[1].acc_bound < (int64_t(1) << 22) ? 1 : 0;
+    // cluster size: enough CTAs to fill the GPU, no fewer than the exact key
+    // chunks need, at most 8, and no CTA without keys
+    const int key_blocks = int((d.L + 63) / 64);
+    const int max_blocks = std::max(1, p->max_keys / 64);
+    const int need = (key_blocks + max_blocks - 1) / max_blocks;
+    int cs = std::max(need, std::min(8, std::max(1, p->num_sms / a.heads)));   // one wave when it can
+    cs = std::max(1, std::min({cs, 8, key_blocks}));
+    if (cs < need) return fail(QX_ERR_UNSUPPORTED, "reassociated attention needs more than 8 key chunks");
+    const int per = (key_blocks + cs - 1) / cs;
+    cs = (key_blocks + per - 1) / per;
+    a.key_splits = cs;
+    a.keys_per_split = per * 64;
+    const int q_tiles = int((d.L + 127) / 128);
+    a.ra_q_per_cta = ((q_tiles + cs - 1) / cs) * 128;
+    QX_CUDA(attn_reassoc_prepare(), "kernel attributes");
+    return QX_OK;
+}
+
 static qx_status build_attn(qx_plan p) {
     const qx_plan_desc &d = p->desc;
     if (d.in_dtype == QX_F32) return build_attn_f32(p);
+    if (d.flags & QX_FLAG_ATTN_REASSOC) return build_attn_reassoc(p);
     const uint64_t H = uint64_t(d.heads);
     p->dp = d.d <= 64 ? 64 : 128;
     p->Lp = int((d.L + 7) / 8 * 8);
@@ -874,7 +997,7 @@ static qx_status pack(qx_plan p, const void *a, const void *b, const void *c, cu
                 return QX_OK;
             }
             QX_CUDA(launch_pack_attn(i32, a, b, c, int(d.heads), int(d.L), int(d.d), p->dp, p->Lp, p->aq, p->ak,
-                                     p->avt, check, d.range_a, d.range_b, d.range_c, p->err,
+                                     p->avt, p->akt, check, d.range_a, d.range_b, d.range_c, p->err,
                                      p->num_sms, st),
                     "operand packing launch");
             return QX_OK;
@@ -921,7 +1044,10 @@ static qx_status run_packed(qx_plan p, void *out, cudaStream_t st) {
                 QX_CUDA(attn_f32_launch(a, st), "attention launch");
                 return QX_OK;
             }
-            QX_CUDA(attn_launch(a, st), "attention launch");
+            if (d.flags & QX_FLAG_ATTN_REASSOC)
+                QX_CUDA(attn_reassoc_launch(a, st), "attention launch");
+            else
+                QX_CUDA(attn_launch(a, st), "attention launch");
             return QX_OK;
         }
     }

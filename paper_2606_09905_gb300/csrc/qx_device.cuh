@@ -343,6 +343,14 @@ __device__ __forceinline__ uint32_t ld_cluster_u32(uint32_t addr) {
     return v;
 }
 
+// Store to shared memory of any CTA of the cluster (an address from
+// cluster_map); fire and forget, made visible by the next cluster barrier.
+__device__ __forceinline__ void st_cluster_v4(uint32_t addr, uint4 v) {
+    asm volatile("st.shared::cluster.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y),
+                 "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
 __device__ __forceinline__ uint4 ld_cluster_v4(uint32_t addr) {
     uint4 v;
     asm volatile("ld.shared::cluster.v4.u32 {%0, %1, %2, %3}, [%4];"

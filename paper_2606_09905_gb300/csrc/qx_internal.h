@@ -77,8 +77,12 @@ struct AttnArgs {
     int *err;
     int L, d, heads;
     int q_tiles, key_splits, keys_per_split;   // key_splits = cluster size (<= 8)
-    int s_shift;              // digit width of the S limbs (integer kind)
+    int s_shift;              // digit width of the S limbs (integer kind); of the
+                              // W digits in the reassociated order
     int o_chunk_kb;           // key-blocks per FP32 chunk of the second product
+    int ra_digits;            // reassociated order: balanced digits of W = K^T V
+    int ra_q_per_cta;         // reassociated order: query rows per CTA (multiple of 128)
+    int ra_fast_cvt;          // reassociated order: phase-2 sums stay below 2^22 in magnitude
 };
 
 }  // namespace qx

@@ -302,15 +302,17 @@ __global__ void __launch_bounds__(256) pack_conv_f32_kernel(const ConvPackF32Arg
 // ------------------------------------------------------- attention operands
 // Q, K, V are heads x L x d.  Q and K become [head][L][dp] FP16 (one head
 // after another, so the rows are simply the heads * L input rows); V becomes
-// [head][dp][Lp] (transposed per head, keys contiguous).
+// [head][dp][Lp] (transposed per head, keys contiguous).  For the
+// reassociated order K is transposed like V instead (k_t set, k unused).
 struct AttnPackArgs {
     const void *Q, *K, *V;
     int heads, L, d, dp, Lp;
     __half *q, *k;          // heads*L x dp each
     __half *vt;             // heads x dp x Lp
+    __half *kt;             // heads x dp x Lp, or null
     RangeCheck cq, ck, cv;
     int *err;
-    int qk_blocks;          // blocks [0, qk_blocks) pack Q and K; the rest transpose V
+    int qk_blocks;          // blocks [0, qk_blocks) pack the row operands; the rest transpose
     int v_tiles_l, v_tiles_c;
 };
 
@@ -324,7 +326,7 @@ __global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
     if (int(blockIdx.x) < p.qk_blocks) {
         const int gpr = p.dp >> 3;
         const int64_t rows = int64_t(p.heads) * p.L;
-        const int64_t items = 2 * rows * gpr;
+        const int64_t items = (p.kt ? 1 : 2) * rows * gpr;   // Q only when K is transposed
         for (int64_t it = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; it < items;
              it += int64_t(p.qk_blocks) * blockDim.x) {
             const int which = int(it / (rows * gpr));
@@ -347,18 +349,22 @@ __global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
         return;
     }
     const int per_head = p.v_tiles_l * p.v_tiles_c;
-    const int hd = (int(blockIdx.x) - p.qk_blocks) / per_head;
-    const int t = int(blockIdx.x) - p.qk_blocks - hd * per_head;
+    int tile_id = int(blockIdx.x) - p.qk_blocks;
+    const bool is_k = tile_id >= p.heads * per_head;    // second half: K^T (reassociated order)
+    if (is_k) tile_id -= p.heads * per_head;
+    const int hd = tile_id / per_head;
+    const int t = tile_id - hd * per_head;
     const int l0 = (t % p.v_tiles_l) * 64;
     const int c0 = (t / p.v_tiles_l) * 64;
-    const T *Vh = V + int64_t(hd) * p.L * p.d;
-    __half *vth = p.vt + int64_t(hd) * p.dp * p.Lp;
+    const T *Vh = (is_k ? K : V) + int64_t(hd) * p.L * p.d;
+    __half *vth = (is_k ? p.kt : p.vt) + int64_t(hd) * p.dp * p.Lp;
+    const RangeCheck &chk = is_k ? p.ck : p.cv;
     for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
         const int lr = i >> 6, cc = i & 63;
         int32_t v = 0;
         if (l0 + lr < p.L && c0 + cc < p.d) {
             v = int32_t(Vh[int64_t(l0 + lr) * p.d + c0 + cc]);
-            p.cv.test(v, p.err);
+            chk.test(v, p.err);
         }
         tile[lr][cc] = v;
     }
@@ -550,8 +556,8 @@ cudaError_t launch_pack_conv_f32(const float *x, const float *w, int n, int c, i
 }
 
 cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int heads, int L,
-                             int d, int dp, int Lp, __half *q, __half *k, __half *vt, int check,
-                             qx_range rq, qx_range rk, qx_range rv, int *err, int num_sms,
+                             int d, int dp, int Lp, __half *q, __half *k, __half *vt, __half *kt,
+                             int check, qx_range rq, qx_range rk, qx_range rv, int *err, int num_sms,
                              cudaStream_t st) {
     AttnPackArgs p;
     p.Q = Q;
@@ -565,17 +571,18 @@ cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void 
     p.q = q;
     p.k = k;
     p.vt = vt;
+    p.kt = kt;
     p.cq = make_check(check, rq);
     p.ck = make_check(check, rk);
     p.cv = make_check(check, rv);
     p.err = err;
-    const int64_t qk_items = int64_t(2) * heads * L * (dp / 8);
+    const int64_t qk_items = int64_t(kt ? 1 : 2) * heads * L * (dp / 8);
     int64_t qk_blocks = (qk_items + 255) / 256;
     if (qk_blocks > int64_t(num_sms) * 4) qk_blocks = int64_t(num_sms) * 4;
     p.qk_blocks = int(qk_blocks);
     p.v_tiles_l = (Lp + 63) / 64;
     p.v_tiles_c = (dp + 63) / 64;
-    const int64_t grid = p.qk_blocks + int64_t(heads) * p.v_tiles_l * p.v_tiles_c;
+    const int64_t grid = p.qk_blocks + int64_t(kt ? 2 : 1) * heads * p.v_tiles_l * p.v_tiles_c;
     if (grid > INT32_MAX) return cudaErrorInvalidValue;
     if (i32) pack_attn_kernel<int32_t><<<grid, 256, 0, st>>>(p);
     else pack_attn_kernel<int16_t><<<grid, 256, 0, st>>>(p);

@@ -23,6 +23,7 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CONTRACT, ERR_OOM, ERR_CUDA, ERR_TIMEO
 OP_GEMM, OP_CONV2D, OP_ATTN, OP_MINMAX, OP_MAXPOOL, OP_AVGPOOL = 0, 1, 2, 3, 4, 5
 I16, I32, F32 = 0, 1, 2
 FLAG_CHECK_RANGES = 1
+FLAG_ATTN_REASSOC = 2         # attention: O = Q (K^T V), integer plans only
 
 # Every function the header declares; the CPU tests check the exports.
 EXPORTS = ("qx_plan_create", "qx_plan_destroy", "qx_plan_query", "qx_plan_info",

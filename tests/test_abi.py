@@ -83,3 +83,28 @@ def test_plan_create_without_device_fails_cleanly(lib):
     with pytest.raises(qx.QxError) as e:
         qx.Plan(qx.gemm_desc(8, 8, 8, (-1, 1), (-1, 1)), device=0)
     assert e.value.status in (qx.ERR_DEVICE, qx.ERR_CUDA)
+
+
+def test_query_reassociated_attention(lib):
+    R = qx.FLAG_ATTN_REASSOC
+    s0, s1 = qx.query(qx.attn_desc(1024, 64, (-7, 7), (-7, 7), (-7, 7), flags=R))
+    # phase 1: one FP32 chunk of K^T V covers all 1024 keys (49 per key term)
+    assert s0["k"] == 1024 and s0["n_chunks"] == 1 and s0["acc_bound"] == 1024 * 49
+    # phase 2: W = K^T V (|W| <= 50176) in two balanced digits, exact over d = 64
+    assert s1["limbs_a"] == 2 and s1["k"] == 64 and s1["acc_bound"] <= 2**24
+    # three digits when max|Q| leaves little room for each digit
+    s1 = qx.query(qx.attn_desc(512, 64, (-1000, 1000), (-20, 20), (-20, 20), flags=R))[1]
+    assert s1["limbs_a"] == 3 and s1["acc_bound"] <= 2**24
+
+
+def test_reassociated_attention_rejects(lib):
+    R = qx.FLAG_ATTN_REASSOC
+    with pytest.raises(qx.QxError) as e:
+        qx.query(qx.attn_desc(64, 64, (0, 0), (0, 0), (0, 0), dtype=qx.F32, flags=R))
+    assert e.value.status == qx.ERR_UNSUPPORTED
+    with pytest.raises(qx.QxError) as e:
+        qx.query(qx.gemm_desc(8, 8, 8, (-1, 1), (-1, 1), flags=R))
+    assert e.value.status == qx.ERR_INVALID_ARG
+    with pytest.raises(qx.QxError) as e:                      # 2048 * 2048 per key term
+        qx.query(qx.attn_desc(1024, 64, (-7, 7), (-2048, 2048), (-2048, 2048), flags=R))
+    assert e.value.status == qx.ERR_CONTRACT

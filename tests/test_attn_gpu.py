@@ -150,6 +150,60 @@ def test_attn_heads_range_check_flags_a_bad_head():
         assert plan.status() == qx.ERR_CONTRACT
 
 
+# ------------------------------------------- reassociated order Q (K^T V)
+def attn_gpu_reassoc(Q, K, V, rq, rk, rv, dtype=qx.I16, flags=0):
+    heads = Q.shape[0] if Q.dim() == 3 else 0
+    L, d = Q.shape[-2:]
+    desc = qx.attn_desc(L, d, rq, rk, rv, dtype=dtype, heads=max(1, heads),
+                        flags=qx.FLAG_ATTN_REASSOC | flags)
+    with qx.Plan(desc) as plan:
+        O = plan.attn(Q.cuda(), K.cuda(), V.cuda())
+        torch.cuda.synchronize()
+        st = plan.status()
+        info = plan.info()
+    return O.cpu().numpy().astype(np.int64), st, info
+
+
+@pytest.mark.parametrize("H,L,d", [(0, 1024, 64), (0, 100, 10), (3, 129, 8), (2, 300, 128),
+                                   (5, 640, 96), (1, 1, 64), (0, 4096, 64), (40, 256, 32)])
+def test_attn_reassoc_matches_oracle(H, L, d):
+    # the oracle computes (Q K^T) V as written; the kernel Q (K^T V): the same integers
+    Q, K, V = inputs.attn_case(L, d, -7, 7, seed=7 * H + L + d, heads=H)
+    ref, _, _ = oracle.attn(Q, K, V)
+    got, st, info = attn_gpu_reassoc(Q, K, V, (-7, 7), (-7, 7), (-7, 7))
+    assert st == qx.OK
+    assert_exact(got, ref, f"reassociated H={H} L={L} d={d} {info}")
+
+
+def test_attn_reassoc_three_digits_and_int32():
+    # max|Q| = 1000 forces W = K^T V into three digits (N = 192)
+    g = torch.Generator().manual_seed(41)
+    Q = torch.randint(-1000, 1001, (2, 512, 64), generator=g, dtype=torch.int32)
+    K = torch.randint(-20, 21, (2, 512, 64), generator=g, dtype=torch.int32)
+    V = torch.randint(-20, 21, (2, 512, 64), generator=g, dtype=torch.int32)
+    ref, _, _ = oracle.attn(Q, K, V)
+    got, st, info = attn_gpu_reassoc(Q, K, V, (-1000, 1000), (-20, 20), (-20, 20), dtype=qx.I32)
+    assert st == qx.OK and info[1]["limbs_a"] == 3
+    assert_exact(got, ref, f"reassociated, 3 digits {info}")
+
+
+def test_attn_reassoc_sampled_large():
+    H, L, d = 32, 2048, 64
+    Q, K, V = inputs.attn_case(L, d, -7, 7, seed=43, heads=H)
+    got, st, _ = attn_gpu_reassoc(Q, K, V, (-7, 7), (-7, 7), (-7, 7))
+    assert st == qx.OK
+    for h in (0, 13, 31):
+        ref, _, _ = oracle.attn(Q[h], K[h], V[h])
+        assert_exact(got[h], ref, f"head {h}")
+
+
+def test_attn_reassoc_range_check_covers_transposed_k():
+    Q, K, V = inputs.attn_case(256, 64, -7, 7, seed=44, heads=2)
+    K[1, 200, 5] = -8
+    _, st, _ = attn_gpu_reassoc(Q, K, V, (-7, 7), (-7, 7), (-7, 7), flags=qx.FLAG_CHECK_RANGES)
+    assert st == qx.ERR_CONTRACT
+
+
 # ------------------------------------------------------------ FP32 (3xTF32)
 def attn_gpu_f32(Q, K, V):
     L, d = Q.shape
