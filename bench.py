@@ -296,6 +296,22 @@ def operators(torch, qx, inputs, dev, only=None):
         r["roofline"] = op_roofline(flops, tensor_peak, nbytes, peaks["hbm_gbs"], r["execute_ms"])
         return r
 
+    def lenet(batch):
+        # LeNet-5 shapes: MACs per image = conv1 6*28*28*25 + conv2 16*10*10*150
+        # + fc 400*120 + 120*84 + 84*10 = 416,520; ops = 2 * MACs
+        macs = 6 * 28 * 28 * 25 + 16 * 10 * 10 * 150 + 400 * 120 + 120 * 84 + 84 * 10
+        ops = 2.0 * macs * batch
+        x, *ws = (t.to(dev) for t in inputs.lenet_case(batch, seed=0))
+        logits = torch.empty((batch, 10), dtype=torch.int32, device=dev)
+        make = lambda: qx.Lenet(batch, (0, 255), [(-7, 7)] * 5, (4, 5, 5, 5), 255)
+        r = op_times(torch, make, lambda net: net.forward(x, ws, logits), ops, 50, dev)
+        r["workload"] = (f"LeNet-5-shaped INT32 pipeline, batch {batch} x 1x32x32, weights in [-7,7], "
+                         f"ReLU + shift + clamp [0,255] between layers; ops = 2 x 416,520 MACs per image")
+        r["images_per_s"] = round(batch / (r["execute_ms"] * 1e-3), 1)
+        nbytes = x.numel() * 4 + sum(w.numel() * 4 for w in ws) + logits.numel() * 4
+        r["roofline"] = op_roofline(ops, peaks["bf16_tflops"], nbytes, peaks["hbm_gbs"], r["execute_ms"])
+        return r
+
     def stream_op(name, make_desc, make_input, call, in_bytes, out_bytes):
         x = make_input().to(dev)
         r = op_times(torch, lambda: qx.Plan(make_desc()), lambda p: call(p, x), 0.0, 50, dev)
@@ -341,6 +357,7 @@ def operators(torch, qx, inputs, dev, only=None):
              "attn_int32": lambda: attn(qx.I32), "attn_fp32": lambda: attn(qx.F32),
              "attn_mh_int16": lambda: attn(qx.I16, H=32, L=2048),
              "attn_mh_fp32": lambda: attn(qx.F32, H=32, L=2048),
+             "lenet_b1": lambda: lenet(1), "lenet_b4096": lambda: lenet(4096),
              "attn_ra_int16": lambda: attn(qx.I16, reassoc=True),
              "attn_mh_ra_int16": lambda: attn(qx.I16, H=32, L=2048, reassoc=True)}
     return {k: f() for k, f in table.items() if only is None or k in only}

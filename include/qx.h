@@ -88,6 +88,14 @@ typedef struct {
  * L * max|K| * max|V| < 2^31 (the entries of K^T V as int32). */
 #define QX_FLAG_ATTN_REASSOC 2u
 
+/* Integer GEMM and Conv2D plans: write min(max(acc, 0) >> rq_shift, rq_hi)
+ * instead of acc -- a ReLU and a requantizing arithmetic right shift,
+ * clamped to [0, rq_hi], applied in the kernel's epilogue, so the output can
+ * feed the next layer under that layer's operand-range contract.  The plan
+ * then requires the exact accumulator to fit int32 (K max|a| max|b| < 2^31,
+ * conv K = c r s), 0 <= rq_shift <= 31 and rq_hi >= 0. */
+#define QX_FLAG_RELU_REQUANT 4u
+
 typedef struct {
     qx_op op;
     qx_dtype in_dtype; /* I16 or I32 operands -> int32 output; F32 -> float */
@@ -113,6 +121,8 @@ typedef struct {
      * and the range contract; head h reads Q[h], K[h], V[h] and writes O[h].
      * 0 and 1 both mean a single head.  At most 65535.  Ignored otherwise. */
     int64_t heads;
+    /* With QX_FLAG_RELU_REQUANT: the right shift and the upper clamp. */
+    int64_t rq_shift, rq_hi;
 } qx_plan_desc;
 
 /* How the plan makes one contraction exact on FP16 tensor cores.  An
@@ -203,6 +213,49 @@ qx_status qx_minmax(qx_plan plan, const void *x, void *result, qx_stream stream)
  * FP32 mean for floats.  x and y are NCHW of the plan's in_dtype (I16, I32
  * or F32). */
 qx_status qx_pool2d(qx_plan plan, const void *x, void *y, qx_stream stream);
+
+/* ------------------------------------------------------------------------
+ * LeNet-shaped INT32 pipeline (Results: the end-to-end "CNN performance"
+ * LeNet run).  The paper names the model only; this executor uses the classic
+ * LeNet-5 layer shapes on N x 1 x 32 x 32 int32 images:
+ *   conv 6@5x5 -> requant -> pool 2x2/2 -> conv 16@5x5 -> requant -> pool 2x2/2
+ *   -> flatten (NCHW order, 400) -> fc 120 -> requant -> fc 84 -> requant
+ *   -> fc 10, raw int32 logits,
+ * where requant(v) = min(max(v, 0) >> shift, act_hi) is applied in the
+ * producing conv / GEMM kernel's epilogue (QX_FLAG_RELU_REQUANT), so every
+ * layer's operands stay inside its range contract.  Each layer is a plan of
+ * this library; the executor owns the seven plans and the activations.
+ * Weights (device, int32, caller-owned): w1 6x1x5x5 and w2 16x6x5x5 (KCRS),
+ * w3 400x120, w4 120x84, w5 84x10 (row-major K x N, y = x w). */
+typedef struct {
+    int64_t batch;              /* images per forward call, >= 1 */
+    qx_range range_x;           /* input pixels */
+    qx_range range_w[5];        /* w1 .. w5 */
+    int64_t shift[4];           /* requantizing shifts after conv1, conv2, fc1, fc2 */
+    int64_t act_hi;             /* activations are clamped to [0, act_hi] */
+    unsigned avg_pool;          /* 0: max pooling; 1: average, floor(sum / 4) */
+} qx_lenet_desc;
+
+typedef struct qx_lenet_s *qx_lenet;
+
+/* Creates the seven layer plans (setup) and one activation buffer on
+ * `device`.  Errors as qx_plan_create, e.g. CONTRACT when a layer's
+ * accumulator could leave int32 under the declared ranges. */
+qx_status qx_lenet_create(const qx_lenet_desc *desc, int device, qx_lenet *out);
+
+/* logits (batch x 10 int32, device) = the pipeline on x (batch x 1 x 32 x 32
+ * int32, device), asynchronous on `stream`: twelve kernel launches (packing +
+ * tensor-core kernel per conv / fc layer, one per pooling layer). */
+qx_status qx_lenet_forward(qx_lenet net, const int32_t *x, const int32_t *w1, const int32_t *w2,
+                           const int32_t *w3, const int32_t *w4, const int32_t *w5,
+                           int32_t *logits, qx_stream stream);
+
+/* Synchronises the device, then returns and clears the first sticky device
+ * error of the seven plans, or QX_OK. */
+qx_status qx_lenet_status(qx_lenet net);
+
+/* Frees the plans and the activations.  NULL is a no-op. */
+qx_status qx_lenet_destroy(qx_lenet net);
 
 /* Synchronises the plan's device, then returns and clears the sticky device
  * error word (QX_ERR_TIMEOUT or QX_ERR_CONTRACT), or QX_OK. */

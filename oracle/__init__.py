@@ -20,6 +20,11 @@ Definitions (paper: Abstract, Methodology paragraph, Table 1, Table 2):
 * ``minmax``  smallest and largest element (Table 2 min/max rows).
 * ``pool2d``  NCHW max / average pooling without padding (Table 2 pooling
   rows); integer averages are floor(window sum / window size).
+* ``requant`` min(max(acc, 0) >> shift, hi): ReLU, arithmetic right shift and
+  clamp between the layers of an integer pipeline.
+* ``lenet``   the LeNet-shaped INT32 pipeline (Results, CNN performance): the
+  classic LeNet-5 layer shapes composed from conv2d, requant, pool2d and
+  gemm above.
 * ``*_f64``   the same three definitions in float64; ``*_absref`` applies them
   to element-wise absolute values, giving the per-element magnitude
   sum |a_k||b_k| that the FP32 tolerance is stated against.
@@ -274,3 +279,32 @@ def pool2d(x, kh: int = 2, kw: int = 2, stride: int = 2, mode: str = "max"):
         y = np.zeros((n, c, P, Q), dtype=np.float64)
         _load().qxo_pool2d_f64(n, c, h, w, kh, kw, stride, is_max, _ptr(a), _ptr(y))
     return y
+
+
+# ------------------------------------------------------ integer pipeline
+def requant(acc, shift: int, hi: int):
+    """ReLU, arithmetic right shift by `shift`, clamp to `hi` (int64)."""
+    a = np.asarray(_np(acc), dtype=np.int64)
+    return np.minimum(np.maximum(a, 0) >> shift, hi)
+
+
+LENET_SHAPES = {            # classic LeNet-5 layer shapes (the paper names only "LeNet")
+    "x": (1, 32, 32), "w1": (6, 1, 5, 5), "w2": (16, 6, 5, 5),
+    "w3": (400, 120), "w4": (120, 84), "w5": (84, 10),
+}
+
+
+def lenet(x, w1, w2, w3, w4, w5, shifts, act_hi: int, pool: str = "max"):
+    """LeNet-shaped INT32 pipeline on N x 1 x 32 x 32 images:
+    conv 6@5x5 -> requant -> pool 2x2/2 -> conv 16@5x5 -> requant -> pool 2x2/2
+    -> flatten (NCHW order, 400) -> fc 120 -> requant -> fc 84 -> requant
+    -> fc 10 (raw int32 logits).  `shifts` are the four requantizing shifts."""
+    x = _np(x)
+    a = requant(conv2d(x, w1), shifts[0], act_hi)
+    a = pool2d(a, 2, 2, 2, pool)
+    a = requant(conv2d(a, w2), shifts[1], act_hi)
+    a = pool2d(a, 2, 2, 2, pool)
+    a = a.reshape(a.shape[0], -1)
+    a = requant(gemm(a, w3)[0], shifts[2], act_hi)
+    a = requant(gemm(a, w4)[0], shifts[3], act_hi)
+    return gemm(a, w5)[0]

@@ -57,6 +57,11 @@ cudaError_t launch_pack_conv(bool i32, const void *x, const void *w, int n, int 
                              int k_out, int r, int s, int Cp, __half *x_planes, __half *w_planes,
                              int nx, int shift_x, int nw, int shift_w, int check, qx_range rx,
                              qx_range rw, int *err, int num_sms, cudaStream_t st);
+cudaError_t launch_pack_patches(bool i32, const void *x, const void *w, int n, int c, int h, int wd,
+                                int k_out, int r, int s, int stride, int pad, int P, int Q, int Kp,
+                                __half *x_planes, __half *w_planes, int nx, int shift_x, int nw,
+                                int shift_w, int check, qx_range rx, qx_range rw, int *err,
+                                int num_sms, cudaStream_t st);
 cudaError_t attn_reassoc_prepare();
 cudaError_t attn_reassoc_launch(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int heads, int L, int d,
@@ -114,6 +119,7 @@ struct qx_plan_s {
     __half *planes_n = nullptr, *planes_m = nullptr;
     float *fplanes_n = nullptr, *fplanes_m = nullptr;   // FP32 kinds
     int Kp = 0, Cp = 0;
+    bool conv_patches = false;                             // conv lowered to explicit patches
     // attention
     AttnArgs attn{};
     int s_shift = 0, max_keys = 0, dp = 0, Lp = 0;
@@ -180,6 +186,27 @@ static qx_status check_device(int device, int *num_sms) {
 }
 
 // Scheme(s) of a descriptor; host only.
+// Integer convs with fewer than 32 input channels are lowered to explicit
+// patches at packing time: an im2col tile carries 64 channels per filter tap,
+// which would be mostly zero padding.
+static bool conv_uses_patches(const qx_plan_desc *d) {
+    return d->c < 32 && d->c * d->r * d->s <= 4096 && d->n * d->c * d->h * d->w < (int64_t(1) << 31);
+}
+
+static int64_t range_mag(qx_range r) { return std::max(r.lo < 0 ? -r.lo : r.lo, r.hi < 0 ? -r.hi : r.hi); }
+
+// ReLU-requantize epilogue: the exact accumulator must be an int32 value.
+static qx_status check_requant(const qx_plan_desc *d, int64_t k_terms) {
+    if (!(d->flags & QX_FLAG_RELU_REQUANT)) return QX_OK;
+    if (d->in_dtype == QX_F32) return fail(QX_ERR_UNSUPPORTED, "requantization is for integer plans");
+    if (d->rq_shift < 0 || d->rq_shift > 31 || d->rq_hi < 0 || d->rq_hi > INT32_MAX)
+        return fail(QX_ERR_INVALID_ARG, "rq_shift must be in [0, 31] and rq_hi in [0, 2^31 - 1]");
+    const __int128 worst = __int128(k_terms) * range_mag(d->range_a) * range_mag(d->range_b);
+    if (worst > INT32_MAX)
+        return fail(QX_ERR_CONTRACT, "requantization needs K max|a| max|b| < 2^31");
+    return QX_OK;
+}
+
 static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, int *s_shift,
                               int *max_keys) {
     if (!d) return fail(QX_ERR_INVALID_ARG, "null descriptor");
@@ -193,6 +220,8 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
         return fail(QX_ERR_INVALID_ARG, "QX_FLAG_ATTN_REASSOC applies to attention plans only");
     if ((d->flags & QX_FLAG_ATTN_REASSOC) && f32)
         return fail(QX_ERR_UNSUPPORTED, "the reassociated attention order is exact for integer plans only");
+    if ((d->flags & QX_FLAG_RELU_REQUANT) && d->op != QX_OP_GEMM && d->op != QX_OP_CONV2D)
+        return fail(QX_ERR_INVALID_ARG, "QX_FLAG_RELU_REQUANT applies to GEMM and conv plans only");
     auto range_ok = [&](qx_range r) {
         if (f32) return true;   // no range contract for FP32 operands
         if (bad_range(r)) return false;
@@ -209,6 +238,10 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
             // N side = A (rows of C), M side = B (columns of C)
             if (!plan_contraction(d->range_a, d->range_b, d->K, &out[0]))
                 return fail(QX_ERR_CONTRACT, "no exact limb scheme for these ranges and K");
+            {
+                const qx_status st = check_requant(d, d->K);
+                if (st != QX_OK) return st;
+            }
             *count = 1;
             return QX_OK;
         }
@@ -239,10 +272,21 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
                 return QX_OK;
             }
             const int64_t Cp = (d->c + 63) / 64 * 64;
+            const int64_t Kc = conv_uses_patches(d) ? (d->c * d->r * d->s + 7) / 8 * 8 : d->r * d->s * Cp;
+            if (conv_uses_patches(d)) {
+                const int64_t P = (d->h + 2 * d->pad - d->r) / d->stride + 1;
+                const int64_t Q = (d->w + 2 * d->pad - d->s) / d->stride + 1;
+                if (d->n * P * Q > INT32_MAX / 2)
+                    return fail(QX_ERR_UNSUPPORTED, "more than 2^30 output pixels");
+            }
             // N side = weights (output channels), M side = x (output pixels)
-            if (!plan_contraction(d->range_b, d->range_a, d->r * d->s * Cp, &out[0]))
+            if (!plan_contraction(d->range_b, d->range_a, Kc, &out[0]))
                 return fail(QX_ERR_CONTRACT, "no exact limb scheme for these ranges");
             if (out[0].m.limbs > 2) return fail(QX_ERR_UNSUPPORTED, "input needs >2 limbs");
+            {
+                const qx_status st = check_requant(d, d->c * d->r * d->s);
+                if (st != QX_OK) return st;
+            }
             *count = 1;
             return QX_OK;
         }
@@ -458,6 +502,9 @@ static qx_status build_gemm(qx_plan p) {
     a.err = p->err;
     a.out_row_stride = d.ldc;
     a.mode = 0;
+    a.rq_on = (d.flags & QX_FLAG_RELU_REQUANT) ? 1 : 0;
+    a.rq_shift = int(d.rq_shift);
+    a.rq_hi = int(d.rq_hi);
     a.m_extent = int(d.N);
     a.n_extent = int(d.M);
     a.kblocks = int((d.K + kBK - 1) / kBK);
@@ -537,9 +584,71 @@ static qx_status build_conv_f32(qx_plan p) {
     return QX_OK;
 }
 
+// Conv on explicit patch planes: the limb GEMM in mode 2 (2-D M-side loads
+// like a GEMM, NCHW stores like a conv).
+static qx_status build_conv_patches(qx_plan p) {
+    const qx_plan_desc &d = p->desc;
+    const Scheme &s = p->scheme[0];
+    const int nw = s.n.limbs, nx = s.m.limbs;
+    const int mr = limb_gemm_rows_per_limb(nw);
+    const int64_t P = (d.h + 2 * d.pad - d.r) / d.stride + 1;
+    const int64_t Q = (d.w + 2 * d.pad - d.s) / d.stride + 1;
+    const int64_t M = d.n * P * Q;
+    p->conv_patches = true;
+    p->Kp = int((d.c * d.r * d.s + 7) / 8 * 8);
+    const size_t x_bytes = size_t(nx) * M * p->Kp * 2;
+    const size_t w_bytes = size_t(nw) * d.k_out * p->Kp * 2;
+    p->ws_bytes = 256 + align256(x_bytes) + align256(w_bytes);
+    QX_CUDA(cudaMalloc(&p->ws, p->ws_bytes), "workspace allocation");
+    p->err = static_cast<int *>(p->ws);
+    p->planes_m = reinterpret_cast<__half *>(static_cast<char *>(p->ws) + 256);
+    p->planes_n = reinterpret_cast<__half *>(static_cast<char *>(p->ws) + 256 + align256(x_bytes));
+    QX_CUDA(cudaMemset(p->err, 0, sizeof(int)), "error word reset");
+
+    MmaArgs &a = p->mma;
+    memset(&a, 0, sizeof a);
+    for (int j = 0; j < nx; ++j) {
+        const uint64_t dims[2] = {uint64_t(p->Kp), uint64_t(M)};
+        const uint64_t str[1] = {uint64_t(p->Kp) * 2};
+        const uint32_t box[2] = {kBK, kBM};
+        qx_status st = encode_tiled(&a.tm_m[j], p->planes_m + size_t(j) * M * p->Kp, 2, dims, str, box);
+        if (st != QX_OK) return st;
+    }
+    {
+        const uint64_t dims[3] = {uint64_t(p->Kp), uint64_t(d.k_out), uint64_t(nw)};
+        const uint64_t str[2] = {uint64_t(p->Kp) * 2, uint64_t(d.k_out) * p->Kp * 2};
+        const uint32_t box[3] = {kBK, uint32_t(mr), uint32_t(nw)};
+        qx_status st = encode_tiled(&a.tm_n, p->planes_n, 3, dims, str, box);
+        if (st != QX_OK) return st;
+    }
+    a.err = p->err;
+    a.out_row_stride = P * Q;
+    a.mode = 2;
+    a.m_extent = int(M);
+    a.n_extent = int(d.k_out);
+    a.kblocks = int((p->Kp + kBK - 1) / kBK);
+    a.chunk_kb = int(s.chunk_kb);
+    a.tiles_m = int((M + kBM - 1) / kBM);
+    a.tiles_n = int((d.k_out + mr - 1) / mr);
+    a.group_n = std::max(1, std::min(16, a.tiles_n));
+    a.shift_n = s.n.shift;
+    a.shift_m = s.m.shift;
+    a.Q = int(Q);
+    a.PQ = int(P * Q);
+    a.k_out = int(d.k_out);
+    a.rq_on = (d.flags & QX_FLAG_RELU_REQUANT) ? 1 : 0;
+    a.rq_shift = int(d.rq_shift);
+    a.rq_hi = int(d.rq_hi);
+    const int tiles = a.tiles_m * a.tiles_n;
+    p->grid = std::max(1, std::min(tiles, p->num_sms));
+    QX_CUDA(limb_gemm_prepare(nw, nx), "kernel attributes");
+    return QX_OK;
+}
+
 static qx_status build_conv(qx_plan p) {
     const qx_plan_desc &d = p->desc;
     if (d.in_dtype == QX_F32) return build_conv_f32(p);
+    if (conv_uses_patches(&d)) return build_conv_patches(p);
     const Scheme &s = p->scheme[0];
     const int nw = s.n.limbs, nx = s.m.limbs;
     const int mr = limb_gemm_rows_per_limb(nw);
@@ -600,6 +709,9 @@ static qx_status build_conv(qx_plan p) {
     a.stride = int(d.stride);
     a.pad = int(d.pad);
     a.k_out = int(d.k_out);
+    a.rq_on = (d.flags & QX_FLAG_RELU_REQUANT) ? 1 : 0;
+    a.rq_shift = int(d.rq_shift);
+    a.rq_hi = int(d.rq_hi);
     const int tiles = a.tiles_m * a.tiles_n;
     p->grid = std::max(1, std::min(tiles, p->num_sms));
     QX_CUDA(limb_gemm_prepare(nw, nx), "kernel attributes");
@@ -977,6 +1089,17 @@ static qx_status pack(qx_plan p, const void *a, const void *b, const void *c, cu
                 return QX_OK;
             }
             const Scheme &s = p->scheme[0];
+            if (p->conv_patches) {
+                const int P = int((d.h + 2 * d.pad - d.r) / d.stride + 1);
+                const int Q = int((d.w + 2 * d.pad - d.s) / d.stride + 1);
+                QX_CUDA(launch_pack_patches(i32, a, b, int(d.n), int(d.c), int(d.h), int(d.w),
+                                            int(d.k_out), int(d.r), int(d.s), int(d.stride),
+                                            int(d.pad), P, Q, p->Kp, p->planes_m, p->planes_n,
+                                            s.m.limbs, s.m.shift, s.n.limbs, s.n.shift, check,
+                                            d.range_a, d.range_b, p->err, p->num_sms, st),
+                        "operand packing launch");
+                return QX_OK;
+            }
             QX_CUDA(launch_pack_conv(i32, a, b, int(d.n), int(d.c), int(d.h), int(d.w),
                                      int(d.k_out), int(d.r), int(d.s), p->Cp, p->planes_m,
                                      p->planes_n, s.m.limbs, s.m.shift, s.n.limbs, s.n.shift, check,

@@ -55,15 +55,18 @@ struct MmaArgs {
     void *out;                // set per call: int32 (exact integer kinds) or float (TF32x3)
     int *err;                 // device error word
     int64_t out_row_stride;   // elements between consecutive N-side rows
-    int mode;                 // 0 = GEMM, 1 = conv (im2col M side, NCHW out)
+    int mode;                 // 0 = GEMM; 1 = conv, im2col M side; 2 = conv on explicit
+                              // patch planes (2-D M side); conv writes NCHW
     int m_extent;             // M-side rows (GEMM: N columns of C; conv: pixels)
     int n_extent;             // N-side rows (GEMM: M rows of C; conv: k_out)
     int kblocks;              // ceil(K / kBK)
     int chunk_kb;             // k-blocks per FP32 accumulation chunk
     int tiles_m, tiles_n, group_n;
     int shift_n, shift_m;     // digit widths of the N-side / M-side limbs
-    // conv geometry (mode 1)
+    // conv geometry (modes 1 and 2)
     int c_blocks, S, Q, PQ, stride, pad, k_out;
+    // output = min(max(acc, 0) >> rq_shift, rq_hi) when rq_on (integer kinds)
+    int rq_on, rq_shift, rq_hi;
 };
 
 // Kernel arguments of the fused attention core.

@@ -1,0 +1,182 @@
+// qx_lenet.cu -- the LeNet-shaped INT32 pipeline executor (paper: Results,
+// "CNN performance": an end-to-end LeNet run on the substrate).  Host code
+// only: it chains plans of this library (two convs and three GEMMs with the
+// ReLU-requantize epilogue, two poolings) on one stream, with every
+// activation in one device allocation made at setup.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdint>
+#include <cstring>
+#include <new>
+
+#include "qx.h"
+
+struct qx_lenet_s {
+    qx_lenet_desc desc{};
+    int device = 0;
+    qx_plan conv1 = nullptr, pool1 = nullptr, conv2 = nullptr, pool2 = nullptr;
+    qx_plan fc1 = nullptr, fc2 = nullptr, fc3 = nullptr;
+    void *act = nullptr;
+    int32_t *a1 = nullptr, *p1 = nullptr, *a2 = nullptr, *p2 = nullptr, *f1 = nullptr, *f2 = nullptr;
+};
+
+namespace {
+
+size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
+
+qx_plan_desc conv_desc(int64_t n, int64_t c, int64_t hw, int64_t k, qx_range rx, qx_range rw,
+                       int64_t shift, int64_t hi) {
+    qx_plan_desc d;
+    memset(&d, 0, sizeof d);
+    d.op = QX_OP_CONV2D;
+    d.in_dtype = QX_I32;
+    d.n = n;
+    d.c = c;
+    d.h = d.w = hw;
+    d.k_out = k;
+    d.r = d.s = 5;
+    d.stride = 1;
+    d.pad = 0;
+    d.range_a = rx;
+    d.range_b = rw;
+    d.flags = QX_FLAG_RELU_REQUANT;
+    d.rq_shift = shift;
+    d.rq_hi = hi;
+    return d;
+}
+
+qx_plan_desc pool_desc(int64_t n, int64_t c, int64_t hw, bool avg) {
+    qx_plan_desc d;
+    memset(&d, 0, sizeof d);
+    d.op = avg ? QX_OP_AVGPOOL : QX_OP_MAXPOOL;
+    d.in_dtype = QX_I32;
+    d.n = n;
+    d.c = c;
+    d.h = d.w = hw;
+    d.r = d.s = 2;
+    d.stride = 2;
+    return d;
+}
+
+qx_plan_desc fc_desc(int64_t m, int64_t n, int64_t k, qx_range ra, qx_range rb, bool rq, int64_t shift,
+                     int64_t hi) {
+    qx_plan_desc d;
+    memset(&d, 0, sizeof d);
+    d.op = QX_OP_GEMM;
+    d.in_dtype = QX_I32;
+    d.M = m;
+    d.N = n;
+    d.K = k;
+    d.range_a = ra;
+    d.range_b = rb;
+    if (rq) {
+        d.flags = QX_FLAG_RELU_REQUANT;
+        d.rq_shift = shift;
+        d.rq_hi = hi;
+    }
+    return d;
+}
+
+void destroy_plans(qx_lenet n) {
+    for (qx_plan *p : {&n->conv1, &n->pool1, &n->conv2, &n->pool2, &n->fc1, &n->fc2, &n->fc3}) {
+        qx_plan_destroy(*p);
+        *p = nullptr;
+    }
+}
+
+}  // namespace
+
+extern "C" {
+
+qx_status qx_lenet_create(const qx_lenet_desc *desc, int device, qx_lenet *out) {
+    if (!out) return QX_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!desc || desc->batch < 1 || desc->act_hi < 0 || desc->batch > (int64_t(1) << 20))
+        return QX_ERR_INVALID_ARG;
+    const int64_t N = desc->batch;
+    const qx_range act{0, desc->act_hi};
+    qx_lenet n = new (std::nothrow) qx_lenet_s();
+    if (!n) return QX_ERR_OOM;
+    n->desc = *desc;
+    n->device = device;
+    qx_status st = QX_OK;
+    const bool avg = desc->avg_pool != 0;
+    auto make = [&](qx_plan *p, const qx_plan_desc &d) {
+        if (st == QX_OK) st = qx_plan_create(&d, device, p);
+    };
+    make(&n->conv1, conv_desc(N, 1, 32, 6, desc->range_x, desc->range_w[0], desc->shift[0], desc->act_hi));
+    make(&n->pool1, pool_desc(N, 6, 28, avg));
+    make(&n->conv2, conv_desc(N, 6, 14, 16, act, desc->range_w[1], desc->shift[1], desc->act_hi));
+    make(&n->pool2, pool_desc(N, 16, 10, avg));
+    make(&n->fc1, fc_desc(N, 120, 400, act, desc->range_w[2], true, desc->shift[2], desc->act_hi));
+    make(&n->fc2, fc_desc(N, 84, 120, act, desc->range_w[3], true, desc->shift[3], desc->act_hi));
+    make(&n->fc3, fc_desc(N, 10, 84, act, desc->range_w[4], false, 0, 0));
+    if (st == QX_OK) {
+        const size_t sizes[6] = {size_t(N) * 6 * 28 * 28, size_t(N) * 6 * 14 * 14, size_t(N) * 16 * 10 * 10,
+                                 size_t(N) * 400, size_t(N) * 120, size_t(N) * 84};
+        size_t total = 0;
+        for (size_t s : sizes) total += align256(s * 4);
+        int prev = 0;
+        cudaGetDevice(&prev);
+        if (cudaSetDevice(device) != cudaSuccess || cudaMalloc(&n->act, total) != cudaSuccess) {
+            st = QX_ERR_OOM;
+        } else {
+            int32_t **slots[6] = {&n->a1, &n->p1, &n->a2, &n->p2, &n->f1, &n->f2};
+            char *base = static_cast<char *>(n->act);
+            for (int i = 0; i < 6; ++i) {
+                *slots[i] = reinterpret_cast<int32_t *>(base);
+                base += align256(sizes[i] * 4);
+            }
+        }
+        cudaSetDevice(prev);
+    }
+    if (st != QX_OK) {
+        destroy_plans(n);
+        if (n->act) cudaFree(n->act);
+        delete n;
+        return st;
+    }
+    *out = n;
+    return QX_OK;
+}
+
+qx_status qx_lenet_forward(qx_lenet n, const int32_t *x, const int32_t *w1, const int32_t *w2,
+                           const int32_t *w3, const int32_t *w4, const int32_t *w5, int32_t *logits,
+                           qx_stream stream) {
+    if (!n || !x || !w1 || !w2 || !w3 || !w4 || !w5 || !logits) return QX_ERR_INVALID_ARG;
+    qx_status st;
+    if ((st = qx_conv2d_gemm(n->conv1, x, w1, n->a1, stream)) != QX_OK) return st;
+    if ((st = qx_pool2d(n->pool1, n->a1, n->p1, stream)) != QX_OK) return st;
+    if ((st = qx_conv2d_gemm(n->conv2, n->p1, w2, n->a2, stream)) != QX_OK) return st;
+    if ((st = qx_pool2d(n->pool2, n->a2, n->p2, stream)) != QX_OK) return st;
+    if ((st = qx_gemm_i32(n->fc1, n->p2, w3, n->f1, stream)) != QX_OK) return st;
+    if ((st = qx_gemm_i32(n->fc2, n->f1, w4, n->f2, stream)) != QX_OK) return st;
+    return qx_gemm_i32(n->fc3, n->f2, w5, logits, stream);
+}
+
+qx_status qx_lenet_status(qx_lenet n) {
+    if (!n) return QX_ERR_INVALID_ARG;
+    qx_status first = QX_OK;
+    for (qx_plan p : {n->conv1, n->pool1, n->conv2, n->pool2, n->fc1, n->fc2, n->fc3}) {
+        const qx_status st = qx_plan_status(p);
+        if (first == QX_OK) first = st;
+    }
+    return first;
+}
+
+qx_status qx_lenet_destroy(qx_lenet n) {
+    if (!n) return QX_OK;
+    destroy_plans(n);
+    if (n->act) {
+        int prev = 0;
+        cudaGetDevice(&prev);
+        cudaSetDevice(n->device);
+        cudaFree(n->act);
+        cudaSetDevice(prev);
+    }
+    delete n;
+    return QX_OK;
+}
+
+}  // extern "C"

@@ -158,7 +158,7 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
                     }
                     uint8_t *st = smem + stage * T::STAGE;
                     mbar_expect_tx(&full[stage], T::STAGE);
-                    if (a.mode == 0) {
+                    if (a.mode != 1) {   // GEMM, or conv on explicit patches
 #pragma unroll
                         for (int j = 0; j < NB; ++j)
                             tma_load_2d(st + j * T::M_TILE, &a.tm_m[j], &full[stage],
@@ -302,6 +302,8 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
                                 (__uint_as_float(v0[x]) + __uint_as_float(v1[x])));
                     }
                 } else {
+                    // 32-row chunks wholly past the N-side extent hold nothing to keep
+                    const int rows_left = a.n_extent - (tn * T::MR + hh * T::RPT);
 #pragma unroll
                     for (int j = 0; j < NB; ++j) {
 #pragma unroll
@@ -309,6 +311,7 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
                             const int sh = i * a.shift_n + j * a.shift_m;
 #pragma unroll
                             for (int p = 0; p < T::RPT / 32; ++p) {
+                                if (p * 32 >= rows_left) continue;
                                 uint32_t v[32];
                                 tmem_ld32(tb + j * T::UN + i * T::MR + p * 32, v);
                                 tmem_wait_ld(v);
@@ -329,9 +332,16 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
             const int mrow = tm * kBM + q * 32 + lane;
             const bool lane_ok = mrow < a.m_extent;
             int64_t lane_off = mrow;
-            if (a.mode == 1) {
+            if (a.mode != 0) {   // conv: pixel mrow of image img, NCHW output
                 const int img = mrow / a.PQ;
                 lane_off = int64_t(img) * a.k_out * a.PQ + (mrow - img * a.PQ);
+            }
+            if constexpr (!T::TF) {
+                if (a.rq_on) {   // ReLU, requantizing shift, clamp
+#pragma unroll
+                    for (int r = 0; r < T::RPT; ++r)
+                        acc[r] = uint32_t(min(max(int32_t(acc[r]), 0) >> a.rq_shift, a.rq_hi));
+                }
             }
             const int nrow0 = tn * T::MR + hh * T::RPT;
             // both output types are 32-bit: store the raw words

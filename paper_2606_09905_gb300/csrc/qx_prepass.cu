@@ -227,6 +227,107 @@ __global__ void __launch_bounds__(256) pack_conv_kernel(const ConvPackArgs p) {
     }
 }
 
+// ------------------------------------------------ conv on explicit patches
+// With few input channels an im2col tile (64 channels per filter tap) would be
+// mostly zero padding, so the packing lowers x to patches instead (the
+// Methodology's "convolution through lowering"): row m = (img, p, q) of the
+// output pixels, element k = (r S + s) c + ch = x[img][ch][p stride - pad + r]
+// [q stride - pad + s], zero outside the image; Kp = c r s rounded up to 8.
+// The weights become rows o with the same k order.
+struct PatchPackArgs {
+    const void *x, *w;
+    int n, c, h, wd, k_out, r, s, stride, pad, P, Q, Kp;
+    __half *x_planes;      // nx planes of (n P Q) x Kp
+    __half *w_planes;      // nw planes of k_out x Kp
+    int shift_x, shift_w;
+    RangeCheck cx, cw;
+    int *err;
+    int x_blocks;          // blocks [0, x_blocks) lower x; the rest pack w
+};
+
+// Per patch element k: the input offset of (ch, r, s) relative to the window
+// corner, and the tap (r, s) for the bounds test, tabled once per block.
+constexpr int kPatchTable = 4096;
+
+template <typename T, int NX, int NW>
+__global__ void __launch_bounds__(256) pack_patches_kernel(const PatchPackArgs p) {
+    pdl_launch_dependents();
+    __shared__ int32_t koff[kPatchTable];
+    __shared__ int32_t ktap[kPatchTable];                // (r << 16) | s, or -1 past c r s
+    const T *X = static_cast<const T *>(p.x);
+    const T *W = static_cast<const T *>(p.w);
+    const int RSC = p.r * p.s * p.c;
+    const int groups = p.Kp >> 3;
+    const int HW = p.h * p.wd;
+    for (int k = threadIdx.x; k < p.Kp; k += blockDim.x) {
+        if (k < RSC) {
+            const int tap = k / p.c;
+            const int ch = k - tap * p.c;
+            const int rr = tap / p.s;
+            const int ss = tap - rr * p.s;
+            koff[k] = ch * HW + rr * p.wd + ss;
+            ktap[k] = (rr << 16) | ss;
+        } else {
+            koff[k] = 0;
+            ktap[k] = -1;
+        }
+    }
+    __syncthreads();
+    if (int(blockIdx.x) < p.x_blocks) {
+        const int PQ = p.P * p.Q;
+        const int M = p.n * PQ;                          // < 2^31 (the plan checks)
+        const int64_t plane_stride = int64_t(M) * p.Kp;
+        for (int64_t it = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; it < int64_t(M) * groups;
+             it += int64_t(p.x_blocks) * blockDim.x) {
+            const int m = int(it / groups);
+            const int g = int(it - int64_t(m) * groups);
+            const int img = m / PQ;
+            const int rem = m - img * PQ;
+            const int oh = rem / p.Q;
+            const int ow = rem - oh * p.Q;
+            const int h0 = oh * p.stride - p.pad;         // window corner
+            const int w0 = ow * p.stride - p.pad;
+            const T *xc = X + int64_t(img) * p.c * HW + h0 * p.wd + w0;
+            int32_t v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int k = 8 * g + e;
+                const int tp = ktap[k];
+                const int ih = h0 + (tp >> 16);
+                const int iw = w0 + (tp & 0xffff);
+                v[e] = 0;
+                if (tp >= 0 && unsigned(ih) < unsigned(p.h) && unsigned(iw) < unsigned(p.wd)) {
+                    v[e] = int32_t(xc[koff[k]]);
+                    p.cx.test(v[e], p.err);
+                }
+            }
+            store_limbs8<NX>(p.x_planes + int64_t(m) * p.Kp + 8 * g, plane_stride, v, p.shift_x);
+        }
+        return;
+    }
+    const int64_t items = int64_t(p.k_out) * groups;
+    const int64_t plane_stride = int64_t(p.k_out) * p.Kp;
+    const int RS = p.r * p.s;
+    for (int64_t it = int64_t(blockIdx.x - p.x_blocks) * blockDim.x + threadIdx.x; it < items;
+         it += int64_t(gridDim.x - p.x_blocks) * blockDim.x) {
+        const int o = int(it / groups);
+        const int g = int(it - int64_t(o) * groups);
+        int32_t v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int k = 8 * g + e;
+            v[e] = 0;
+            if (k < RSC) {
+                const int tap = k / p.c;
+                const int ch = k - tap * p.c;
+                v[e] = int32_t(W[(int64_t(o) * p.c + ch) * RS + tap]);
+                p.cw.test(v[e], p.err);
+            }
+        }
+        store_limbs8<NW>(p.w_planes + int64_t(o) * p.Kp + 8 * g, plane_stride, v, p.shift_w);
+    }
+}
+
 // -------------------------------------------------------- conv, FP32 kind
 // x (NCHW float) -> big and small TF32 planes, NHWC, channels padded to Cp
 // (a multiple of 32, one 128-byte row); w (KCRS) -> (k, r, s, Cp) planes.
@@ -526,6 +627,57 @@ cudaError_t launch_pack_conv(bool i32, const void *x, const void *w, int n, int 
     if (w_blocks < 1) w_blocks = 1;
     const int grid = p.x_blocks + w_blocks;
     return i32 ? pack_conv_t<int32_t>(nx, nw, p, grid, st) : pack_conv_t<int16_t>(nx, nw, p, grid, st);
+}
+
+template <typename T>
+static cudaError_t pack_patches_t(int nx, int nw, const PatchPackArgs &p, int grid, cudaStream_t st) {
+#define QX_PP(A_, B_)                                                                  \
+    if (nx == A_ && nw == B_) {                                                        \
+        pack_patches_kernel<T, A_, B_><<<grid, 256, 0, st>>>(p);                       \
+        return cudaGetLastError();                                                     \
+    }
+    QX_PP(1, 1) QX_PP(1, 2) QX_PP(1, 3) QX_PP(1, 4) QX_PP(2, 1) QX_PP(2, 2) QX_PP(2, 4)
+#undef QX_PP
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_pack_patches(bool i32, const void *x, const void *w, int n, int c, int h, int wd,
+                                int k_out, int r, int s, int stride, int pad, int P, int Q, int Kp,
+                                __half *x_planes, __half *w_planes, int nx, int shift_x, int nw,
+                                int shift_w, int check, qx_range rx, qx_range rw, int *err,
+                                int num_sms, cudaStream_t st) {
+    PatchPackArgs p;
+    p.x = x;
+    p.w = w;
+    p.n = n;
+    p.c = c;
+    p.h = h;
+    p.wd = wd;
+    p.k_out = k_out;
+    p.r = r;
+    p.s = s;
+    p.stride = stride;
+    p.pad = pad;
+    p.P = P;
+    p.Q = Q;
+    p.Kp = Kp;
+    p.x_planes = x_planes;
+    p.w_planes = w_planes;
+    p.shift_x = shift_x;
+    p.shift_w = shift_w;
+    p.cx = make_check(check, rx);
+    p.cw = make_check(check, rw);
+    p.err = err;
+    const int64_t x_items = int64_t(n) * P * Q * (Kp / 8);
+    int64_t x_blocks = (x_items + 255) / 256;
+    if (x_blocks > int64_t(num_sms) * 8) x_blocks = int64_t(num_sms) * 8;
+    p.x_blocks = int(x_blocks < 1 ? 1 : x_blocks);
+    const int64_t w_items = int64_t(k_out) * (Kp / 8);
+    int w_blocks = int((w_items + 255) / 256);
+    if (w_blocks > num_sms) w_blocks = num_sms;
+    if (w_blocks < 1) w_blocks = 1;
+    return i32 ? pack_patches_t<int32_t>(nx, nw, p, p.x_blocks + w_blocks, st)
+               : pack_patches_t<int16_t>(nx, nw, p, p.x_blocks + w_blocks, st);
 }
 
 cudaError_t launch_pack_conv_f32(const float *x, const float *w, int n, int c, int h, int wd,

@@ -68,6 +68,17 @@ def attn_case_f32(L: int, d: int, seed: int, heads: int = 0):
     return tuple(normal(shape, g) for _ in range(3))
 
 
+def lenet_case(batch: int, seed: int, x_hi: int = 255, w_mag: int = 7):
+    """LeNet-shaped INT32 pipeline operands: images N x 1 x 32 x 32 uniform in
+    [0, x_hi] (pixels), then w1 6x1x5x5, w2 16x6x5x5, w3 400x120, w4 120x84,
+    w5 84x10, each uniform in [-w_mag, w_mag]; all int32."""
+    g = _gen(seed)
+    x = int_uniform((batch, 1, 32, 32), 0, x_hi, g, torch.int32)
+    shapes = ((6, 1, 5, 5), (16, 6, 5, 5), (400, 120), (120, 84), (84, 10))
+    ws = tuple(int_uniform(sh, -w_mag, w_mag, g, torch.int32) for sh in shapes)
+    return (x,) + ws
+
+
 @dataclass(frozen=True)
 class Workload:
     name: str

@@ -24,13 +24,15 @@ OP_GEMM, OP_CONV2D, OP_ATTN, OP_MINMAX, OP_MAXPOOL, OP_AVGPOOL = 0, 1, 2, 3, 4, 
 I16, I32, F32 = 0, 1, 2
 FLAG_CHECK_RANGES = 1
 FLAG_ATTN_REASSOC = 2         # attention: O = Q (K^T V), integer plans only
+FLAG_RELU_REQUANT = 4         # GEMM / conv: out = min(max(acc, 0) >> rq_shift, rq_hi)
 
 # Every function the header declares; the CPU tests check the exports.
 EXPORTS = ("qx_plan_create", "qx_plan_destroy", "qx_plan_query", "qx_plan_info",
            "qx_gemm_i16_i32", "qx_gemm_i32", "qx_conv2d_gemm", "qx_attn_core",
            "qx_pack", "qx_run_packed", "qx_plan_status", "qx_status_string",
            "qx_last_error", "qx_version", "qx_gemm_i16_i32_noalloc", "qx_minmax",
-           "qx_pool2d")
+           "qx_pool2d", "qx_lenet_create", "qx_lenet_forward", "qx_lenet_status",
+           "qx_lenet_destroy")
 
 
 class QxError(RuntimeError):
@@ -43,6 +45,11 @@ class Range(ctypes.Structure):
     _fields_ = [("lo", ctypes.c_int64), ("hi", ctypes.c_int64)]
 
 
+class LenetDesc(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int64), ("range_x", Range), ("range_w", Range * 5),
+                ("shift", ctypes.c_int64 * 4), ("act_hi", ctypes.c_int64), ("avg_pool", ctypes.c_uint)]
+
+
 class PlanDesc(ctypes.Structure):
     _fields_ = [("op", ctypes.c_int), ("in_dtype", ctypes.c_int),
                 ("M", ctypes.c_int64), ("N", ctypes.c_int64), ("K", ctypes.c_int64),
@@ -52,7 +59,8 @@ class PlanDesc(ctypes.Structure):
                 ("s", ctypes.c_int64), ("stride", ctypes.c_int64), ("pad", ctypes.c_int64),
                 ("L", ctypes.c_int64), ("d", ctypes.c_int64),
                 ("range_a", Range), ("range_b", Range), ("range_c", Range),
-                ("flags", ctypes.c_uint), ("heads", ctypes.c_int64)]
+                ("flags", ctypes.c_uint), ("heads", ctypes.c_int64),
+                ("rq_shift", ctypes.c_int64), ("rq_hi", ctypes.c_int64)]
 
 
 class SchemeInfo(ctypes.Structure):
@@ -100,6 +108,10 @@ def load() -> ctypes.CDLL:
             "qx_pool2d": ([P, V, V, V], ctypes.c_int),
             "qx_gemm_i16_i32_noalloc": ([ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, Range,
                                          Range, ctypes.c_uint, V, V, V, V, V], ctypes.c_int),
+            "qx_lenet_create": ([ctypes.POINTER(LenetDesc), ctypes.c_int, ctypes.POINTER(P)], ctypes.c_int),
+            "qx_lenet_forward": ([P, V, V, V, V, V, V, V, V], ctypes.c_int),
+            "qx_lenet_status": ([P], ctypes.c_int),
+            "qx_lenet_destroy": ([P], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -121,15 +133,27 @@ def _rng(r) -> Range:
     return Range(int(r[0]), int(r[1]))
 
 
-def gemm_desc(M, N, K, range_a, range_b, dtype=I16, lda=0, ldb=0, ldc=0, flags=0) -> PlanDesc:
+def _requant(flags, requant):
+    """requant = (shift, hi) adds QX_FLAG_RELU_REQUANT; None leaves it off."""
+    if requant is None:
+        return flags, 0, 0
+    shift, hi = requant
+    return flags | FLAG_RELU_REQUANT, shift, hi
+
+
+def gemm_desc(M, N, K, range_a, range_b, dtype=I16, lda=0, ldb=0, ldc=0, flags=0,
+              requant=None) -> PlanDesc:
+    flags, sh, hi = _requant(flags, requant)
     return PlanDesc(op=OP_GEMM, in_dtype=dtype, M=M, N=N, K=K, lda=lda, ldb=ldb, ldc=ldc,
-                    range_a=_rng(range_a), range_b=_rng(range_b), flags=flags)
+                    range_a=_rng(range_a), range_b=_rng(range_b), flags=flags, rq_shift=sh, rq_hi=hi)
 
 
-def conv_desc(n, c, h, w, k_out, r, s, stride, pad, range_x, range_w, dtype=I16, flags=0) -> PlanDesc:
+def conv_desc(n, c, h, w, k_out, r, s, stride, pad, range_x, range_w, dtype=I16, flags=0,
+              requant=None) -> PlanDesc:
+    flags, sh, hi = _requant(flags, requant)
     return PlanDesc(op=OP_CONV2D, in_dtype=dtype, n=n, c=c, h=h, w=w, k_out=k_out, r=r, s=s,
                     stride=stride, pad=pad, range_a=_rng(range_x), range_b=_rng(range_w),
-                    flags=flags)
+                    flags=flags, rq_shift=sh, rq_hi=hi)
 
 
 def attn_desc(L, d, range_q, range_k, range_v, dtype=I16, flags=0, heads=1) -> PlanDesc:
@@ -326,3 +350,59 @@ class Plan:
         po = _ptr(O, out_dt, shape, "O")
         _check(load().qx_attn_core(self.handle, pq, pk, pv, po, _stream(stream)), "qx_attn_core")
         return O
+
+
+# ------------------------------------------------------- LeNet pipeline
+LENET_WEIGHT_SHAPES = ((6, 1, 5, 5), (16, 6, 5, 5), (400, 120), (120, 84), (84, 10))
+
+
+class Lenet:
+    """The LeNet-shaped INT32 pipeline executor (seven plans + activations,
+    created once).  forward(x, weights) -> batch x 10 int32 logits."""
+
+    def __init__(self, batch, range_x, ranges_w, shifts, act_hi, avg_pool=False, device=None):
+        lib = load()
+        if device is None:
+            device = torch.cuda.current_device()
+        self.device = device
+        self.batch = int(batch)
+        d = LenetDesc(batch=self.batch, range_x=_rng(range_x), act_hi=int(act_hi),
+                      avg_pool=1 if avg_pool else 0)
+        for i, r in enumerate(ranges_w):
+            d.range_w[i] = _rng(r)
+        for i, sh in enumerate(shifts):
+            d.shift[i] = int(sh)
+        self.desc = d
+        h = ctypes.c_void_p()
+        _check(lib.qx_lenet_create(ctypes.byref(d), device, ctypes.byref(h)), "qx_lenet_create")
+        self.handle = h
+
+    def forward(self, x, weights, logits=None, stream=None):
+        if logits is None:
+            logits = torch.empty((self.batch, 10), dtype=torch.int32, device=x.device)
+        px = _ptr(x, torch.int32, (self.batch, 1, 32, 32), "x")
+        pw = [_ptr(w, torch.int32, shp, f"w{i + 1}") for i, (w, shp) in
+              enumerate(zip(weights, LENET_WEIGHT_SHAPES))]
+        po = _ptr(logits, torch.int32, (self.batch, 10), "logits")
+        _check(load().qx_lenet_forward(self.handle, px, *pw, po, _stream(stream)), "qx_lenet_forward")
+        return logits
+
+    def status(self) -> int:
+        return int(load().qx_lenet_status(self.handle))
+
+    def close(self):
+        if getattr(self, "handle", None):
+            load().qx_lenet_destroy(self.handle)
+            self.handle = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

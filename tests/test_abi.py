@@ -43,9 +43,10 @@ def test_version_and_strings(lib):
 
 def test_struct_layouts_match_header():
     # qx_plan_desc: 2 ints, 17 int64, 3 ranges (2 x int64), 1 unsigned (+pad),
-    # then the int64 head count
-    assert ctypes.sizeof(qx.PlanDesc) == 8 + 17 * 8 + 3 * 16 + 8 + 8
+    # then the int64 head count and the two requantization fields
+    assert ctypes.sizeof(qx.PlanDesc) == 8 + 17 * 8 + 3 * 16 + 8 + 3 * 8
     assert qx.PlanDesc.heads.offset == 8 + 17 * 8 + 3 * 16 + 8
+    assert qx.PlanDesc.rq_hi.offset == qx.PlanDesc.heads.offset + 16
     assert ctypes.sizeof(qx.SchemeInfo) == 5 * 4 + 4 + 4 * 8
 
 

@@ -146,3 +146,34 @@ def test_conv_f32_integer_values_exact():
     got, st = conv_gpu_f32(x.float(), w.float(), 1, 1)
     assert st == qx.OK
     assert (got == oracle.conv2d(x, w, 1, 1)).all()
+
+
+# ------------------------------------- few input channels (explicit patches)
+@pytest.mark.parametrize("shape,stride,pad", [
+    ((64, 1, 32, 32, 6, 5, 5), 1, 0),         # LeNet conv1
+    ((64, 6, 14, 14, 16, 5, 5), 1, 0),        # LeNet conv2
+    ((3, 31, 9, 9, 33, 3, 3), 1, 1),
+    ((2, 2, 11, 7, 130, 3, 2), 2, 1),
+])
+def test_conv_explicit_patches(shape, stride, pad):
+    n, c, h, wd, k, r, s = shape
+    x, w = inputs.conv_case(n, c, h, wd, k, r, s, -255, 255, seed=sum(shape) + stride, dtype=torch.int32)
+    ref = oracle.conv2d(x, w, stride, pad)
+    got, st, info = conv_gpu(x, w, stride, pad, (-255, 255), (-255, 255), dtype=qx.I32)
+    assert st == qx.OK
+    assert_exact(got, ref, f"conv {shape} s{stride} p{pad} {info}")
+
+
+# ------------------------------------------------ ReLU-requantize epilogue
+@pytest.mark.parametrize("c", [6, 64])      # explicit patches and im2col-on-load
+def test_conv_requant_epilogue(c):
+    x, w = inputs.conv_case(4, c, 12, 12, 20, 3, 3, -255, 255, seed=c, dtype=torch.int32)
+    desc = qx.conv_desc(4, c, 12, 12, 20, 3, 3, 1, 1, (-255, 255), (-255, 255), dtype=qx.I32,
+                        requant=(9, 1000))
+    with qx.Plan(desc) as plan:
+        y = plan.conv2d(x.cuda(), w.cuda())
+        torch.cuda.synchronize()
+        assert plan.status() == qx.OK
+    want = oracle.requant(oracle.conv2d(x, w, 1, 1), 9, 1000)
+    assert 0 < (want == 1000).sum() < want.size and (want == 0).any()   # both clamps exercised
+    assert_exact(y.cpu().numpy().astype(np.int64), want, f"conv requant c={c}")

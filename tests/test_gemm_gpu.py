@@ -209,3 +209,15 @@ def test_full_smul24_operand_range_int32():
     got, st, _ = gemm_gpu(A, B, r, r, dtype=qx.I32)
     assert st == qx.OK
     assert_exact(got, wrap32(ref), "smul24 range")
+
+
+def test_gemm_requant_epilogue():
+    A, B = inputs.gemm_case(300, 130, 200, -255, 255, seed=61, dtype=torch.int32)
+    desc = qx.gemm_desc(300, 130, 200, (-255, 255), (-255, 255), dtype=qx.I32, requant=(8, 5000))
+    with qx.Plan(desc) as plan:
+        C = plan.gemm_i32(A.cuda(), B.cuda())
+        torch.cuda.synchronize()
+        assert plan.status() == qx.OK
+    want = oracle.requant(oracle.gemm(A, B)[0], 8, 5000)
+    assert (want == 5000).any() and (want == 0).any()
+    assert_exact(C.cpu().numpy().astype(np.int64), want, "gemm requant")

@@ -313,3 +313,40 @@ def test_pool_2x2_reshape_identity():
     ref = x.reshape(3, 2, 3, 2, 4, 2).max(axis=(3, 5))
     assert (oracle.pool2d(x, 2, 2, 2, "max") == ref).all()
     assert (oracle.pool2d(np.full((1, 1, 4, 4), -7), 2, 2, 2, "avg") == -7).all()
+
+
+# ------------------------------------------------------ integer pipeline
+def test_requant_closed_form():
+    got = oracle.requant(np.array([-5, 0, 7, 1000, 2**20, -2**30]), 2, 100)
+    assert got.tolist() == [0, 0, 1, 100, 100, 0]
+    assert oracle.requant(np.array([3, 4, 5]), 0, 4).tolist() == [3, 4, 4]
+
+
+def test_requant_commutes_with_max_pooling():
+    # requant is monotone non-decreasing, so it commutes with taking a maximum
+    rng = np.random.default_rng(5)
+    x = rng.integers(-5000, 5000, size=(2, 3, 8, 6))
+    a = oracle.pool2d(oracle.requant(x, 3, 200), 2, 2, 2, "max")
+    b = oracle.requant(oracle.pool2d(x, 2, 2, 2, "max"), 3, 200)
+    assert (a == b).all()
+
+
+def test_lenet_pass_through_network():
+    # Centre-tap convolutions and identity fully connected layers carry one
+    # channel straight through: with no shift and a high clamp the ten logits
+    # all equal the sum of the 5 x 5 map left after the two crops and poolings,
+    # computed here with plain numpy slicing (no conv or GEMM code).
+    rng = np.random.default_rng(6)
+    x = rng.integers(0, 100, size=(3, 1, 32, 32))
+    w1 = np.zeros((6, 1, 5, 5), dtype=np.int64); w1[0, 0, 2, 2] = 1
+    w2 = np.zeros((16, 6, 5, 5), dtype=np.int64); w2[0, 0, 2, 2] = 1
+    w3 = np.zeros((400, 120), dtype=np.int64); w3[np.arange(120), np.arange(120)] = 1
+    w4 = np.zeros((120, 84), dtype=np.int64); w4[np.arange(84), np.arange(84)] = 1
+    w5 = np.ones((84, 10), dtype=np.int64)
+    logits = oracle.lenet(x, w1, w2, w3, w4, w5, (0, 0, 0, 0), 10**6)
+    m = x[:, 0, 2:30, 2:30]                                 # conv1 centre tap
+    m = m.reshape(3, 14, 2, 14, 2).max(axis=(2, 4))         # pool1
+    m = m[:, 2:12, 2:12]                                    # conv2 centre tap
+    m = m.reshape(3, 5, 2, 5, 2).max(axis=(2, 4))           # pool2
+    want = m.reshape(3, -1).sum(axis=1)
+    assert logits.shape == (3, 10) and (logits == want[:, None]).all()
