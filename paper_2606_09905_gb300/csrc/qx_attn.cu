@@ -175,12 +175,75 @@ __device__ __forceinline__ void drain_after_abort(const Bars &b, int issued_kv) 
     mbar_wait_drain(b.q, 0);
 }
 
-// Cluster reduction: CTA `rank` adds its slice of the 128 query rows over all
+// Cluster reduction of the key splits, by pushing.  The 128 query rows are
+// owned round the cluster, rows_per = ceil(128 / cs) per CTA.  After a cluster
+// barrier (every CTA is past its main loop, so every receive buffer is idle)
+// each CTA stores each of its partial rows into the owner's receive buffer
+// [source rank][row - owner's first row][pitch words] with fire-and-forget
+// distributed-shared-memory stores; after a second barrier the owner adds the
+// cs copies in rank order and writes its rows of O.  No atomics, the same
+// order on every run.
+__device__ __forceinline__ int owned_rows(int cs) { return (kQTile + cs - 1) / cs; }
+
+// Cluster address of element (row, col) of this CTA's partial in the owner's buffer.
+__device__ __forceinline__ uint32_t push_addr(uint32_t recv_saddr, int row, int col, int pitch, int cs) {
+    const int rows_per = owned_rows(cs);
+    const int owner = row / rows_per;
+    const int slot = int(cluster_rank()) * rows_per + (row - owner * rows_per);
+    return cluster_map(recv_saddr, uint32_t(owner)) + uint32_t(slot * pitch + col) * 4u;
+}
+
+template <bool FLOAT>
+__device__ __forceinline__ void owner_reduce_store(const uint32_t *recv, int pitch, int cs, int qt, int hd,
+                                                   const AttnArgs &a) {
+    const int rows_per = owned_rows(cs);
+    const int j0 = int(cluster_rank()) * rows_per;
+    const int nrows = min(min(kQTile - j0, rows_per), a.L - qt * kQTile - j0);
+    if (nrows <= 0) return;
+    uint32_t *out = static_cast<uint32_t *>(a.out) + (int64_t(hd) * a.L + int64_t(qt) * kQTile + j0) * a.d;
+    if ((a.d & 3) == 0) {
+        const int groups = a.d >> 2;
+        for (int idx = threadIdx.x; idx < nrows * groups; idx += blockDim.x) {
+            const int jj = idx / groups;
+            const int c = 4 * (idx - jj * groups);
+            uint4 acc = *reinterpret_cast<const uint4 *>(recv + jj * pitch + c);
+            for (int src = 1; src < cs; ++src) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(recv + (src * rows_per + jj) * pitch + c);
+                if constexpr (FLOAT) {
+                    acc.x = __float_as_uint(__uint_as_float(acc.x) + __uint_as_float(v.x));
+                    acc.y = __float_as_uint(__uint_as_float(acc.y) + __uint_as_float(v.y));
+                    acc.z = __float_as_uint(__uint_as_float(acc.z) + __uint_as_float(v.z));
+                    acc.w = __float_as_uint(__uint_as_float(acc.w) + __uint_as_float(v.w));
+                } else {
+                    acc.x += v.x;
+                    acc.y += v.y;
+                    acc.z += v.z;
+                    acc.w += v.w;
+                }
+            }
+            *reinterpret_cast<uint4 *>(out + int64_t(jj) * a.d + c) = acc;
+        }
+        return;
+    }
+    for (int idx = threadIdx.x; idx < nrows * a.d; idx += blockDim.x) {
+        const int jj = idx / a.d;
+        const int c = idx - jj * a.d;
+        uint32_t acc = recv[jj * pitch + c];
+        for (int src = 1; src < cs; ++src) {
+            const uint32_t v = recv[(src * rows_per + jj) * pitch + c];
+            if constexpr (FLOAT) acc = __float_as_uint(__uint_as_float(acc) + __uint_as_float(v));
+            else acc += v;
+        }
+        out[int64_t(jj) * a.d + c] = acc;
+    }
+}
+// Cluster reduction used by the FP32 kernel (measured faster there than
+// pushing: its threads hold columns, not rows): CTA `rank` adds its slice of the 128 query rows over all
 // `cs` CTAs (rank order) and writes O rows qt*128 + j of head `hd`.  part is
 // [128][pitch] (int32 or float words, pitch a multiple of 4).  Rows of O are
 // written four columns at a time when d is a multiple of 4.
 template <bool FLOAT>
-__device__ __forceinline__ void cluster_reduce_store(const void *part, int pitch, int cs, int qt, int hd,
+__device__ __forceinline__ void cluster_pull_reduce_store(const void *part, int pitch, int cs, int qt, int hd,
                                                      const AttnArgs &a) {
     const uint32_t rank = cluster_rank();
     const int rows = (kQTile + cs - 1) / cs;
@@ -289,6 +352,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
     pdl_wait();   // packed operands come from the kernel launched just before
 
     bool ok = true;
+    uint32_t keep[64];                                   // converters: partial O row (cluster case)
     if (warp == kProducerWarp) {
         // ---------------------------------------------------------- TMA loads
         if (lane == 0 && nb > 0) {
@@ -451,8 +515,7 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
             __syncwarp();
             if (lane == 0) mbar_arrive(&bar.sready[i]);
         }
-        // ------------------------ this CTA's partial O -> shared memory
-        // (the K / V^T ring is idle once the last O product has completed)
+        // ------------------- this CTA's partial O -> registers or global memory
         const int last = nb - 1;
         const bool have = ok && nb > 0 &&
                           mbar_wait(&bar.o_done[last % nsb], uint32_t((last / nsb) & 1), bar.abort_flag, a.err);
@@ -463,8 +526,10 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
         int32_t *orow = static_cast<int32_t *>(a.out) + (int64_t(hd) * a.L + q) * a.d;
         const bool vec = (a.d & 3) == 0;
         const int cols = dp / 2;                         // output columns of this warp
-#pragma unroll 1
-        for (int c0 = h * cols; c0 < (h + 1) * cols; c0 += 32) {
+#pragma unroll
+        for (int cc = 0; cc < 64; cc += 32) {
+            if (cc >= cols) break;
+            const int c0 = h * cols + cc;
             uint32_t lo[32], hi[32];
             if (have) {
                 tmem_ld32(tOlo + lane_off + uint32_t(c0), lo);
@@ -472,7 +537,6 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
                 tmem_wait_ld(lo);
                 tmem_wait_ld(hi);
             }
-            int32_t *dst = part + row * pitch + c0;
 #pragma unroll
             for (int x = 0; x < 32; x += 4) {
                 uint4 w = make_uint4(0u, 0u, 0u, 0u);
@@ -487,7 +551,10 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
                           (uint32_t(__float2int_rn(__uint_as_float(hi[x + 3]))) << a.s_shift);
                 }
                 if (cs > 1) {
-                    *reinterpret_cast<uint4 *>(dst + x) = w;
+                    keep[cc + x] = w.x;
+                    keep[cc + x + 1] = w.y;
+                    keep[cc + x + 2] = w.z;
+                    keep[cc + x + 3] = w.w;
                 } else if (q < a.L) {
                     const int c = c0 + x;
                     if (vec && c + 3 < a.d) {
@@ -506,9 +573,17 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
     tc_fence_before();
     __syncthreads();
     if (cs > 1) {
-        cluster_sync();                                  // every partial is in place
-        cluster_reduce_store<false>(part, pitch, cs, qt, hd, a);
-        cluster_sync();                                  // peers are done reading
+        cluster_sync();                                  // every CTA is past its main loop
+        if (warp < kProducerWarp) {
+            const int rowq = (warp & 3) * 32 + lane;
+            const int c0 = (warp >> 2) * (dp / 2);
+            const uint32_t dst = push_addr(smem_addr(part), rowq, c0, pitch, cs);
+#pragma unroll
+            for (int c = 0; c < 64; c += 4)
+                if (c < dp / 2) st_cluster_v4(dst + uint32_t(c) * 4u, make_uint4(keep[c], keep[c + 1], keep[c + 2], keep[c + 3]));
+        }
+        cluster_sync();                                  // every partial row has arrived
+        owner_reduce_store<false>(reinterpret_cast<const uint32_t *>(part), pitch, cs, qt, hd, a);
     }
     if (warp == kIssuerWarp) {
         tc_fence_after();
@@ -691,7 +766,7 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
     __syncthreads();
     if (cs > 1) {
         cluster_sync();
-        cluster_reduce_store<true>(part, kDp32, cs, qt, hd, a);
+        cluster_pull_reduce_store<true>(part, kDp32, cs, qt, hd, a);
         cluster_sync();
     }
     if (warp == 4) {
