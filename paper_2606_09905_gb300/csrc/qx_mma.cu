@@ -67,7 +67,12 @@ struct TileCfg {
     static constexpr int BK_ELEMS = TF ? kBK32 : kBK;                     // K per 128-byte row
     static constexpr int BAR_BYTES = 256;
     static constexpr int SMEM = STAGES * STAGE + BAR_BYTES + 1024;
-    static constexpr int THREADS = 320;
+    // warp 0: M-side TMA producer; warp 1: TMEM + MMA issue; warps 2-9:
+    // epilogue; warp 10: N-side TMA producer.  One thread needs a few hundred
+    // cycles to issue a TMA load, so two producer threads keep a k-block's
+    // loads within its MMA time.
+    static constexpr int THREADS = 352;
+    static constexpr int N_PRODUCER_WARP = 10;
     static_assert(UN % 16 == 0 && UN >= 16 && UN <= 256, "MMA N out of range");
     static_assert(TMEM_NEED <= 512, "accumulators exceed tensor memory");
     static_assert(RPT % 32 == 0, "epilogue works in 32-column TMEM loads");
@@ -87,7 +92,7 @@ __device__ __forceinline__ void tile_coords(int t, const MmaArgs &a, int &tm, in
 }
 
 template <int NA, int NB, int KIND>
-__global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant__ MmaArgs a) {
+__global__ void __launch_bounds__(352, 1) limb_gemm_kernel(const __grid_constant__ MmaArgs a) {
     using T = TileCfg<NA, NB, KIND>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -111,7 +116,7 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
         if (NB > 1) tma_prefetch(&a.tm_m[1]);
         tma_prefetch(&a.tm_n);
         for (int s = 0; s < T::STAGES; ++s) {
-            mbar_init(&full[s], 1);
+            mbar_init(&full[s], 2);          // one arrive.expect_tx per producer
             mbar_init(&empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -157,7 +162,7 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
                         break;
                     }
                     uint8_t *st = smem + stage * T::STAGE;
-                    mbar_expect_tx(&full[stage], T::STAGE);
+                    mbar_expect_tx(&full[stage], NB * T::M_TILE);
                     if (a.mode != 1) {   // GEMM, or conv on explicit patches
 #pragma unroll
                         for (int j = 0; j < NB; ++j)
@@ -175,8 +180,6 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
                                                oh * a.stride - a.pad, img, uint16_t(s),
                                                uint16_t(r));
                     }
-                    tma_load_3d(st + NB * T::M_TILE, &a.tm_n, &full[stage], kb * T::BK_ELEMS,
-                                tn * T::MR, 0);
                     ++issued;
                     if (++stage == T::STAGES) {
                         stage = 0;
@@ -262,6 +265,39 @@ __global__ void __launch_bounds__(320, 1) limb_gemm_kernel(const __grid_constant
                 // MMAs already issued must finish before TMEM is released.
                 tc_commit(tail);
                 mbar_wait_drain(tail, 0);
+            }
+        }
+    } else if (warp == T::N_PRODUCER_WARP) {
+        if (lane == 0) {
+            // ---------------------------------------- TMA producer, N side
+            int stage = 0;
+            uint32_t phase = 0;
+            long long issued = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+                int tm, tn;
+                tile_coords(t, a, tm, tn);
+                for (int kb = 0; kb < a.kblocks; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, a.err)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(&full[stage], T::N_TILE);
+                    tma_load_3d(smem + stage * T::STAGE + NB * T::M_TILE, &a.tm_n, &full[stage],
+                                kb * T::BK_ELEMS, tn * T::MR, 0);
+                    ++issued;
+                    if (++stage == T::STAGES) {
+                        stage = 0;
+                        phase ^= 1;
+                    }
+                }
+            }
+            if (*abort_flag) {
+                // Let every copy already issued land before shared memory goes.
+                for (int s = 0; s < T::STAGES; ++s) {
+                    const long long uses = issued / T::STAGES + (s < issued % T::STAGES ? 1 : 0);
+                    if (uses > 0) mbar_wait_drain(&full[s], uint32_t((uses - 1) & 1));
+                }
             }
         }
     } else {
