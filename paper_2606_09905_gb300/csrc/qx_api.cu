@@ -222,6 +222,8 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
         return fail(QX_ERR_UNSUPPORTED, "the reassociated attention order is exact for integer plans only");
     if ((d->flags & QX_FLAG_RELU_REQUANT) && d->op != QX_OP_GEMM && d->op != QX_OP_CONV2D)
         return fail(QX_ERR_INVALID_ARG, "QX_FLAG_RELU_REQUANT applies to GEMM and conv plans only");
+    if ((d->flags & QX_FLAG_RELU_REQUANT) && f32)
+        return fail(QX_ERR_UNSUPPORTED, "requantization is for integer plans");
     auto range_ok = [&](qx_range r) {
         if (f32) return true;   // no range contract for FP32 operands
         if (bad_range(r)) return false;

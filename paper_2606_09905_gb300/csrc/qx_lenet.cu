@@ -12,6 +12,10 @@
 
 #include "qx.h"
 
+namespace qx {
+void set_last_error(const char *msg);   // qx_api.cu
+}  // namespace qx
+
 struct qx_lenet_s {
     qx_lenet_desc desc{};
     int device = 0;
@@ -90,10 +94,15 @@ void destroy_plans(qx_lenet n) {
 extern "C" {
 
 qx_status qx_lenet_create(const qx_lenet_desc *desc, int device, qx_lenet *out) {
-    if (!out) return QX_ERR_INVALID_ARG;
-    *out = nullptr;
-    if (!desc || desc->batch < 1 || desc->act_hi < 0 || desc->batch > (int64_t(1) << 20))
+    if (!out) {
+        qx::set_last_error("null executor output");
         return QX_ERR_INVALID_ARG;
+    }
+    *out = nullptr;
+    if (!desc || desc->batch < 1 || desc->act_hi < 0 || desc->batch > (int64_t(1) << 20)) {
+        qx::set_last_error("LeNet descriptor: need 1 <= batch <= 2^20 and act_hi >= 0");
+        return QX_ERR_INVALID_ARG;
+    }
     const int64_t N = desc->batch;
     const qx_range act{0, desc->act_hi};
     qx_lenet n = new (std::nothrow) qx_lenet_s();
@@ -120,6 +129,8 @@ qx_status qx_lenet_create(const qx_lenet_desc *desc, int device, qx_lenet *out) 
         int prev = 0;
         cudaGetDevice(&prev);
         if (cudaSetDevice(device) != cudaSuccess || cudaMalloc(&n->act, total) != cudaSuccess) {
+            cudaGetLastError();
+            qx::set_last_error("LeNet activation allocation failed");
             st = QX_ERR_OOM;
         } else {
             int32_t **slots[6] = {&n->a1, &n->p1, &n->a2, &n->p2, &n->f1, &n->f2};
@@ -144,7 +155,10 @@ qx_status qx_lenet_create(const qx_lenet_desc *desc, int device, qx_lenet *out) 
 qx_status qx_lenet_forward(qx_lenet n, const int32_t *x, const int32_t *w1, const int32_t *w2,
                            const int32_t *w3, const int32_t *w4, const int32_t *w5, int32_t *logits,
                            qx_stream stream) {
-    if (!n || !x || !w1 || !w2 || !w3 || !w4 || !w5 || !logits) return QX_ERR_INVALID_ARG;
+    if (!n || !x || !w1 || !w2 || !w3 || !w4 || !w5 || !logits) {
+        qx::set_last_error("null executor, operand or output pointer");
+        return QX_ERR_INVALID_ARG;
+    }
     qx_status st;
     if ((st = qx_conv2d_gemm(n->conv1, x, w1, n->a1, stream)) != QX_OK) return st;
     if ((st = qx_pool2d(n->pool1, n->a1, n->p1, stream)) != QX_OK) return st;

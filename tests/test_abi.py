@@ -109,3 +109,43 @@ def test_reassociated_attention_rejects(lib):
     with pytest.raises(qx.QxError) as e:                      # 2048 * 2048 per key term
         qx.query(qx.attn_desc(1024, 64, (-7, 7), (-2048, 2048), (-2048, 2048), flags=R))
     assert e.value.status == qx.ERR_CONTRACT
+
+
+def test_requant_flag_validation(lib):
+    R = (4, 255)
+    with pytest.raises(qx.QxError) as e:                     # integer plans only
+        qx.query(qx.conv_desc(1, 8, 8, 8, 4, 3, 3, 1, 1, (0, 0), (0, 0), dtype=qx.F32, requant=R))
+    assert e.value.status == qx.ERR_UNSUPPORTED
+    with pytest.raises(qx.QxError) as e:                     # not an attention option
+        d = qx.attn_desc(64, 64, (-7, 7), (-7, 7), (-7, 7))
+        d.flags |= qx.FLAG_RELU_REQUANT
+        qx.query(d)
+    assert e.value.status == qx.ERR_INVALID_ARG
+    with pytest.raises(qx.QxError) as e:                     # shift out of range
+        qx.query(qx.gemm_desc(8, 8, 8, (-1, 1), (-1, 1), dtype=qx.I32, requant=(32, 1)))
+    assert e.value.status == qx.ERR_INVALID_ARG
+    # K max|a| max|b| = 64 * 2^11 * 2^12 = 2^29 fits; doubling K * |b| twice does not
+    qx.query(qx.gemm_desc(8, 8, 64, (-2**11, 2**11), (-2**12, 2**12), dtype=qx.I32, requant=(0, 5)))
+    with pytest.raises(qx.QxError) as e:
+        qx.query(qx.gemm_desc(8, 8, 256, (-2**11, 2**11), (-2**12, 2**12), dtype=qx.I32, requant=(0, 5)))
+    assert e.value.status == qx.ERR_CONTRACT
+
+
+def test_conv_few_channels_is_lowered_to_patches(lib):
+    # c r s rounded up to 8 is the contraction length of the explicit patches
+    s = qx.query(qx.conv_desc(4096, 1, 32, 32, 6, 5, 5, 1, 0, (0, 255), (-7, 7), dtype=qx.I32))[0]
+    assert s["k"] == 32
+    s = qx.query(qx.conv_desc(8, 6, 14, 14, 16, 5, 5, 1, 0, (0, 255), (-7, 7), dtype=qx.I32))[0]
+    assert s["k"] == 152
+    # 64 channels keep im2col-on-load: 9 taps x 64 channels
+    s = qx.query(qx.conv_desc(8, 64, 56, 56, 128, 3, 3, 1, 1, (-255, 255), (-255, 255)))[0]
+    assert s["k"] == 576
+
+
+def test_lenet_create_rejects_bad_arguments(lib):
+    with pytest.raises(qx.QxError) as e:
+        qx.Lenet(0, (0, 255), [(-7, 7)] * 5, (4, 5, 5, 5), 255, device=0)
+    assert e.value.status == qx.ERR_INVALID_ARG
+    with pytest.raises(qx.QxError) as e:
+        qx.Lenet(8, (0, 255), [(-7, 7)] * 5, (4, 5, 5, 5), -1, device=0)
+    assert e.value.status == qx.ERR_INVALID_ARG
