@@ -47,13 +47,6 @@ def workload_name():
             f"values i.i.d. uniform [{LO},{HI}]")
 
 
-def _env_int(name, default):
-    try:
-        return int(os.environ.get(name, default))
-    except ValueError:
-        return default
-
-
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -411,7 +404,8 @@ def sweep(args):
 
 # -------------------------------------------------------------------- main
 def run_reference(args):
-    rank = _env_int("RANK", 0)
+    from paper_2606_09905_gb300 import replicas
+    rank, _, _ = replicas.rank_world_local()
     if rank != 0:
         return 0
     steps, warmup = args.steps, args.warmup
@@ -445,11 +439,9 @@ def run_qx(args):
 
     from paper_2606_09905_gb300 import _build
     _build.build()
-    from paper_2606_09905_gb300 import inputs, qx
+    from paper_2606_09905_gb300 import inputs, qx, replicas
 
-    world = _env_int("WORLD_SIZE", 1)
-    rank = _env_int("RANK", 0)
-    local = _env_int("LOCAL_RANK", 0)
+    rank, world, local = replicas.rank_world_local()
     if world != args.gpus and world > 1:
         raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE {world}")
     torch.cuda.set_device(local)
@@ -457,11 +449,8 @@ def run_qx(args):
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
 
-    def barrier():
-        if world > 1:
-            dist.barrier()
-
-    A, B = inputs.gemm_case(M, N, K, LO, HI, seed=rank)
+    barrier = replicas.barrier
+    A, B = inputs.gemm_case(M, N, K, LO, HI, seed=replicas.replica_seed(rank))
     dA, dB = A.to(dev), B.to(dev)
     C = torch.empty((M, N), dtype=torch.int32, device=dev)
     desc = qx.gemm_desc(M, N, K, (LO, HI), (LO, HI))
@@ -499,11 +488,7 @@ def run_qx(args):
     torch.cuda.synchronize(dev)
     barrier()
     clocks = sampler.stop()
-    ms_total = t_start.elapsed_time(t_stop)
-    if world > 1:
-        tt = torch.tensor([ms_total], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_total = float(tt.item())
+    ms_total = replicas.max_over_ranks(t_start.elapsed_time(t_stop), dev)
     ms_step = ms_total / args.steps
     kernel_ms = statistics.mean(m[0].elapsed_time(m[1]) for m in marks)
     pack_ms = statistics.mean(s.elapsed_time(m[0]) for s, m in zip(starts, marks))
@@ -512,7 +497,7 @@ def run_qx(args):
         raise SystemExit(f"device status {st} after the timed region")
 
     ops = 2.0 * M * N * K
-    value = world * ops / (ms_step * 1e-3) / 1e12
+    value = replicas.whole_job_rate(ops, ms_step * 1e-3, world) / 1e12
 
     # -------------------------------------------- end to end, host buffers
     # Every step copies its inputs from pinned host memory, runs the GEMM
@@ -567,11 +552,8 @@ def run_qx(args):
     e2e_ms = e0.elapsed_time(e1) / e2e_steps
     if not (all(torch.equal(hC[0], h) for h in hC[1:]) and torch.equal(hC[0], dC2[0].cpu())):
         raise SystemExit("pipelined end-to-end results disagree")
-    if world > 1:
-        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
-    e2e = {"value": world * ops / (e2e_ms * 1e-3) / 1e12, "unit": "TOPS",
+    e2e_ms = replicas.max_over_ranks(e2e_ms, dev)
+    e2e = {"value": replicas.whole_job_rate(ops, e2e_ms * 1e-3, world) / 1e12, "unit": "TOPS",
            "h2d_bytes_per_step": hA.numel() * 2 + hB.numel() * 2,
            "d2h_bytes_per_step": hC[0].numel() * 4, "ms_per_step": e2e_ms,
            "pipeline": f"H2D / GEMM / D2H on three streams, {NSET} buffer sets; bound by the host link"}
