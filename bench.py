@@ -173,14 +173,21 @@ def event_pair(torch):
     return torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
 
 
+PER_GRAPH = 10                                   # calls per graph for the execute time
+
+
 def op_times(torch, make_plan, call, ops, reps, dev):
     """Setup / cached steady-state / execute-only times of one operator, as the
     paper separates them (Methodology; Table 2 QPU-C and QPU-E columns):
       setup    plan creation plus the first call, host wall clock;
       cached   host wall clock of one call on a warm plan, synchronised;
-      execute  device time of one call: the call captured once in a CUDA
-               graph and replayed back to back between CUDA events, so no
-               host launch cost is included."""
+      execute  device time per call: PER_GRAPH calls captured back to back
+               in one CUDA graph, the graph replayed between CUDA events, the
+               time divided by the calls, so neither host launch cost nor
+               the graph's own launch is included;
+      execute_1  the same with one call per graph (each replay then adds the
+               graph launch, a few microseconds, which dominates small
+               problems)."""
     torch.cuda.synchronize(dev)
     t0 = time.perf_counter()
     plan = make_plan()
@@ -196,23 +203,29 @@ def op_times(torch, make_plan, call, ops, reps, dev):
         call(plan)
         torch.cuda.synchronize(dev)
         cached.append((time.perf_counter() - t0) * 1e3)
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph):
-        call(plan)
-    graph.replay()
-    torch.cuda.synchronize(dev)
-    s, e = event_pair(torch)
-    s.record()
-    for _ in range(reps):
+    def graph_ms(per_graph):
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            for _ in range(per_graph):
+                call(plan)
         graph.replay()
-    e.record()
-    e.synchronize()
-    x = s.elapsed_time(e) / reps
+        torch.cuda.synchronize(dev)
+        s, e = event_pair(torch)
+        s.record()
+        for _ in range(reps):
+            graph.replay()
+        e.record()
+        e.synchronize()
+        del graph
+        return s.elapsed_time(e) / (reps * per_graph)
+
+    x1 = graph_ms(1)
+    x = graph_ms(PER_GRAPH)
     st = plan.status()
-    del graph
     plan.close()
     c = statistics.median(cached)
     return {"setup_ms": round(setup_ms, 3), "cached_ms": round(c, 4), "execute_ms": round(x, 4),
+            "execute_1_ms": round(x1, 4),
             "cached_gops": round(ops / (c * 1e-3) / 1e9, 1),
             "execute_gops": round(ops / (x * 1e-3) / 1e9, 1), "status": st}
 
@@ -375,8 +388,6 @@ def sweep(args):
               (8192, 8192, 8192, 500)]
     for (m, n, k, r) in shapes:
         for dt, tdt in ((qx.I16, torch.int16), (qx.I32, torch.int32)):
-            if m == 8192 and dt == qx.I32:
-                continue
             tag = f"gemm{m}x{n}x{k}_{'i16' if dt == qx.I16 else 'i32'}"
             if only is not None and tag not in only:
                 continue
@@ -384,10 +395,21 @@ def sweep(args):
             A, B = A.to(dev), B.to(dev)
             C = torch.empty((m, n), dtype=torch.int32, device=dev)
             fn = "gemm_i16_i32" if dt == qx.I16 else "gemm_i32"
+            reps = 20 if m >= 4096 else 100
             res = op_times(torch, lambda: qx.Plan(qx.gemm_desc(m, n, k, (-r, r), (-r, r), dtype=dt)),
-                           lambda p: getattr(p, fn)(A, B, C), 2.0 * m * n * k,
-                           20 if m >= 4096 else 100, dev)
-            res.update(workload=f"{tag} [-{r},{r}]")
+                           lambda p: getattr(p, fn)(A, B, C), 2.0 * m * n * k, reps, dev)
+            with qx.Plan(qx.gemm_desc(m, n, k, (-r, r), (-r, r), dtype=dt)) as p:
+                fused = p.fused
+            res.update(workload=f"{tag} [-{r},{r}]", path="fused" if fused else "prepass")
+            if m * n * k <= 2048**3:
+                # the other path on the same problem, for the record
+                alt = qx.FLAG_PREPASS if fused else qx.FLAG_FUSED_CONVERT
+                other = op_times(torch, lambda: qx.Plan(qx.gemm_desc(m, n, k, (-r, r), (-r, r), dtype=dt,
+                                                                     flags=alt)),
+                                 lambda p: getattr(p, fn)(A, B, C), 2.0 * m * n * k, reps, dev)
+                res["other_path"] = {"path": "prepass" if fused else "fused",
+                                     "cached_ms": other["cached_ms"], "execute_ms": other["execute_ms"],
+                                     "execute_1_ms": other["execute_1_ms"], "status": other["status"]}
             mlimb = qx.query(qx.gemm_desc(m, n, k, (-r, r), (-r, r), dtype=dt))[0]["mma_per_kstep"]
             esz = 2 if dt == qx.I16 else 4
             res["roofline"] = op_roofline(mlimb * 2.0 * m * n * k, peaks["bf16_tflops"],

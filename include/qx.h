@@ -96,6 +96,19 @@ typedef struct {
  * conv K = c r s), 0 <= rq_shift <= 31 and rq_hi >= 0. */
 #define QX_FLAG_RELU_REQUANT 4u
 
+/* Integer GEMM plans: how the operands reach the tensor cores.  By default
+ * (or with QX_FLAG_PREPASS) a packing pre-pass writes the FP16 limb planes
+ * into the workspace and the tensor-core kernel reads them by TMA: two
+ * launches, the faster path at every size measured.  QX_FLAG_FUSED_CONVERT
+ * selects the fused path: one kernel reads A and B as they are and splits
+ * them into FP16 limbs in shared memory (one launch, no limb planes in
+ * device memory); it requires lda and ldb to be multiples of 8 elements for
+ * I16 and of 4 for I32 (rows 16-byte aligned), else plan creation returns
+ * QX_ERR_UNSUPPORTED.  Both paths give the same bits.  qx_pack /
+ * qx_run_packed always take the two-kernel path. */
+#define QX_FLAG_FUSED_CONVERT 8u
+#define QX_FLAG_PREPASS 16u
+
 typedef struct {
     qx_op op;
     qx_dtype in_dtype; /* I16 or I32 operands -> int32 output; F32 -> float */
@@ -244,8 +257,9 @@ typedef struct qx_lenet_s *qx_lenet;
 qx_status qx_lenet_create(const qx_lenet_desc *desc, int device, qx_lenet *out);
 
 /* logits (batch x 10 int32, device) = the pipeline on x (batch x 1 x 32 x 32
- * int32, device), asynchronous on `stream`: twelve kernel launches (packing +
- * tensor-core kernel per conv / fc layer, one per pooling layer). */
+ * int32, device), asynchronous on `stream`: at most twelve kernel launches
+ * (packing + tensor-core kernel per conv layer, one launch per pooling layer,
+ * one or two per fc layer as its plan picks the fused or the pre-pass path). */
 qx_status qx_lenet_forward(qx_lenet net, const int32_t *x, const int32_t *w1, const int32_t *w2,
                            const int32_t *w3, const int32_t *w4, const int32_t *w5,
                            int32_t *logits, qx_stream stream);
@@ -261,6 +275,12 @@ qx_status qx_lenet_destroy(qx_lenet net);
  * error word (QX_ERR_TIMEOUT or QX_ERR_CONTRACT), or QX_OK. */
 qx_status qx_plan_status(qx_plan plan);
 
+/* 1 if the plan's execution call runs the fused single-kernel GEMM (operands
+ * converted to limbs inside the tensor-core kernel), 0 if it runs the packing
+ * pre-pass and then the tensor-core kernel (every non-GEMM plan), -1 for a
+ * NULL plan.  See QX_FLAG_FUSED_CONVERT. */
+int qx_plan_fused(qx_plan plan);
+
 /* Allocation-free INT16 GEMM.  The paper has no counterpart; this entry
  * point exists for callers that cannot call cudaMalloc when they multiply:
  * code running inside an allocator or memory-pool callback (allocating there
@@ -274,8 +294,10 @@ qx_status qx_plan_status(qx_plan plan);
  * 16-byte aligned device pointers on the current device, asynchronous on
  * `stream`; the scheme follows from range_a / range_b as in a plan, and
  * flags takes QX_FLAG_CHECK_RANGES.
- *   - Problems whose planes exceed the scratch (about 24 MiB of operands at
- *     2048^3) return QX_ERR_UNSUPPORTED and launch nothing.
+ *   - Problems whose limb planes exceed the scratch (beyond about 2048^3)
+ *     run the fused single-kernel GEMM (see QX_FLAG_FUSED_CONVERT), which
+ *     needs no planes; it requires K and N to be multiples of 8, otherwise
+ *     the call returns QX_ERR_UNSUPPORTED and launches nothing.
  *   - The first call on a device looks up the scratch's device address
  *     (cudaGetSymbolAddress); make that first call before any stream capture.
  *   - Every call on a device shares the scratch and leaves its planes in it;

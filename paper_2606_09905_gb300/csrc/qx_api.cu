@@ -30,8 +30,12 @@ void scheme_to_info(const Scheme &s, qx_scheme_info *o);
 // kernels
 bool limb_gemm_supported(int na, int nb);
 int limb_gemm_rows_per_limb(int na);
-cudaError_t limb_gemm_prepare(int na, int nb);
+int limb_gemm_pick_rows(int na, int64_t m_extent, int64_t n_extent, int num_sms);
+cudaError_t limb_gemm_prepare(int na, int nb, int mr);
 cudaError_t limb_gemm_launch(int na, int nb, const MmaArgs &a, int grid, cudaStream_t stream);
+bool fused_gemm_packed_ok(int na, int shift_n, int nb, int shift_m, bool values_fit_int16);
+cudaError_t fused_gemm_prepare(int na, int nb, bool i32, bool pk);
+cudaError_t fused_gemm_launch(int na, int nb, bool i32, bool pk, const MmaArgs &a, int grid, cudaStream_t stream);
 cudaError_t tf32x3_prepare();
 cudaError_t tf32x3_launch(const MmaArgs &a, int grid, cudaStream_t stream);
 cudaError_t launch_pack_conv_f32(const float *x, const float *w, int n, int c, int h, int wd,
@@ -116,10 +120,14 @@ struct qx_plan_s {
     // GEMM / conv
     MmaArgs mma{};
     int grid = 0;
+    MmaArgs fmma{};                                        // GEMM, fused path (default tile height)
+    int fgrid = 0;
     __half *planes_n = nullptr, *planes_m = nullptr;
     float *fplanes_n = nullptr, *fplanes_m = nullptr;   // FP32 kinds
     int Kp = 0, Cp = 0;
     bool conv_patches = false;                             // conv lowered to explicit patches
+    bool fused = false;                                    // GEMM: conversion inside the kernel
+    bool fused_packed = false;                             // ... on packed int16 pairs
     // attention
     AttnArgs attn{};
     int s_shift = 0, max_keys = 0, dp = 0, Lp = 0;
@@ -224,6 +232,10 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
         return fail(QX_ERR_INVALID_ARG, "QX_FLAG_RELU_REQUANT applies to GEMM and conv plans only");
     if ((d->flags & QX_FLAG_RELU_REQUANT) && f32)
         return fail(QX_ERR_UNSUPPORTED, "requantization is for integer plans");
+    if ((d->flags & (QX_FLAG_FUSED_CONVERT | QX_FLAG_PREPASS)) && d->op != QX_OP_GEMM)
+        return fail(QX_ERR_INVALID_ARG, "QX_FLAG_FUSED_CONVERT and QX_FLAG_PREPASS apply to GEMM plans only");
+    if ((d->flags & QX_FLAG_FUSED_CONVERT) && (d->flags & QX_FLAG_PREPASS))
+        return fail(QX_ERR_INVALID_ARG, "QX_FLAG_FUSED_CONVERT and QX_FLAG_PREPASS exclude each other");
     auto range_ok = [&](qx_range r) {
         if (f32) return true;   // no range contract for FP32 operands
         if (bad_range(r)) return false;
@@ -469,11 +481,26 @@ struct DeviceScope {
 };
 
 // ------------------------------------------------------------ plan build
+// Rows of A and B start on 16-byte boundaries (given 16-byte aligned bases).
+static bool gemm_rows_aligned(const qx_plan_desc &d) {
+    const int64_t per16 = d.in_dtype == QX_I32 ? 4 : 8;
+    return d.lda % per16 == 0 && d.ldb % per16 == 0;
+}
+
+// Whether a GEMM plan converts its operands inside the tensor-core kernel.
+// Only on request: measured on GB300 at every Table 1 size, the pre-pass
+// path is faster.  The pre-pass converts each element once, spread over all
+// SMs at close to the copy bandwidth; in the fused kernel every CTA converts
+// the whole K extent of its A rows and B columns itself (each A row block
+// once per column tile, each B column block once per row tile), and the
+// conversion, not the tensor cores, sets its pace.
+static bool gemm_uses_fused(const qx_plan_desc &d) { return (d.flags & QX_FLAG_FUSED_CONVERT) != 0; }
+
 static qx_status build_gemm(qx_plan p) {
     const qx_plan_desc &d = p->desc;
     const Scheme &s = p->scheme[0];
     const int na = s.n.limbs, nb = s.m.limbs;
-    const int mr = limb_gemm_rows_per_limb(na);
+    const int mr = limb_gemm_pick_rows(na, d.N, d.M, p->num_sms);
     p->Kp = int((d.K + 7) / 8 * 8);
     const size_t a_bytes = size_t(na) * d.M * p->Kp * 2;
     const size_t b_bytes = size_t(nb) * d.N * p->Kp * 2;
@@ -515,10 +542,33 @@ static qx_status build_gemm(qx_plan p) {
     a.tiles_n = int((d.M + mr - 1) / mr);
     a.shift_n = s.n.shift;
     a.shift_m = s.m.shift;
+    a.mr = mr;
     const int tiles = a.tiles_m * a.tiles_n;
     p->grid = std::max(1, std::min(tiles, p->num_sms));
     a.group_n = tile_group(p->grid, a.tiles_n, nb, na, mr);
-    QX_CUDA(limb_gemm_prepare(na, nb), "kernel attributes");
+    QX_CUDA(limb_gemm_prepare(na, nb, mr), "kernel attributes");
+    // fused conversion: the default tile height; raw operands are set per call
+    MmaArgs &f = p->fmma;
+    f = a;
+    f.mr = limb_gemm_rows_per_limb(na);
+    f.tiles_n = int((d.M + f.mr - 1) / f.mr);
+    const int ftiles = f.tiles_m * f.tiles_n;
+    p->fgrid = std::max(1, std::min(ftiles, p->num_sms));
+    f.group_n = tile_group(p->fgrid, f.tiles_n, nb, na, f.mr);
+    f.lda = d.lda;
+    f.ldb = d.ldb;
+    f.K = int(d.K);
+    f.chk = (d.flags & QX_FLAG_CHECK_RANGES) ? 1 : 0;
+    f.lo_a = d.range_a.lo;
+    f.hi_a = d.range_a.hi;
+    f.lo_b = d.range_b.lo;
+    f.hi_b = d.range_b.hi;
+    p->fused = gemm_uses_fused(d);
+    auto fits16 = [](qx_range r) { return r.lo >= -32768 && r.hi <= 32767; };
+    p->fused_packed = fused_gemm_packed_ok(na, s.n.shift, nb, s.m.shift,
+                                           fits16(d.range_a) && fits16(d.range_b));
+    if (p->fused)
+        QX_CUDA(fused_gemm_prepare(na, nb, d.in_dtype == QX_I32, p->fused_packed), "kernel attributes");
     return QX_OK;
 }
 
@@ -572,6 +622,7 @@ static qx_status build_conv_f32(qx_plan p) {
     a.chunk_kb = a.kblocks;
     a.tiles_m = int((a.m_extent + kBM - 1) / kBM);
     a.tiles_n = int((d.k_out + 127) / 128);
+    a.mr = 128;
     a.group_n = std::max(1, std::min(16, a.tiles_n));
     a.c_blocks = p->Cp / kBK32;
     a.S = int(d.s);
@@ -592,10 +643,10 @@ static qx_status build_conv_patches(qx_plan p) {
     const qx_plan_desc &d = p->desc;
     const Scheme &s = p->scheme[0];
     const int nw = s.n.limbs, nx = s.m.limbs;
-    const int mr = limb_gemm_rows_per_limb(nw);
     const int64_t P = (d.h + 2 * d.pad - d.r) / d.stride + 1;
     const int64_t Q = (d.w + 2 * d.pad - d.s) / d.stride + 1;
     const int64_t M = d.n * P * Q;
+    const int mr = limb_gemm_pick_rows(nw, M, d.k_out, p->num_sms);
     p->conv_patches = true;
     p->Kp = int((d.c * d.r * d.s + 7) / 8 * 8);
     const size_t x_bytes = size_t(nx) * M * p->Kp * 2;
@@ -641,9 +692,10 @@ static qx_status build_conv_patches(qx_plan p) {
     a.rq_on = (d.flags & QX_FLAG_RELU_REQUANT) ? 1 : 0;
     a.rq_shift = int(d.rq_shift);
     a.rq_hi = int(d.rq_hi);
+    a.mr = mr;
     const int tiles = a.tiles_m * a.tiles_n;
     p->grid = std::max(1, std::min(tiles, p->num_sms));
-    QX_CUDA(limb_gemm_prepare(nw, nx), "kernel attributes");
+    QX_CUDA(limb_gemm_prepare(nw, nx, mr), "kernel attributes");
     return QX_OK;
 }
 
@@ -653,9 +705,9 @@ static qx_status build_conv(qx_plan p) {
     if (conv_uses_patches(&d)) return build_conv_patches(p);
     const Scheme &s = p->scheme[0];
     const int nw = s.n.limbs, nx = s.m.limbs;
-    const int mr = limb_gemm_rows_per_limb(nw);
     const int64_t P = (d.h + 2 * d.pad - d.r) / d.stride + 1;
     const int64_t Q = (d.w + 2 * d.pad - d.s) / d.stride + 1;
+    const int mr = limb_gemm_pick_rows(nw, d.n * P * Q, d.k_out, p->num_sms);
     p->Cp = int((d.c + 63) / 64 * 64);
     const size_t x_bytes = size_t(nx) * d.n * d.h * d.w * p->Cp * 2;
     const size_t w_bytes = size_t(nw) * d.k_out * d.r * d.s * p->Cp * 2;
@@ -714,9 +766,10 @@ static qx_status build_conv(qx_plan p) {
     a.rq_on = (d.flags & QX_FLAG_RELU_REQUANT) ? 1 : 0;
     a.rq_shift = int(d.rq_shift);
     a.rq_hi = int(d.rq_hi);
+    a.mr = mr;
     const int tiles = a.tiles_m * a.tiles_n;
     p->grid = std::max(1, std::min(tiles, p->num_sms));
-    QX_CUDA(limb_gemm_prepare(nw, nx), "kernel attributes");
+    QX_CUDA(limb_gemm_prepare(nw, nx, mr), "kernel attributes");
     return QX_OK;
 }
 
@@ -971,6 +1024,10 @@ qx_status qx_plan_create(const qx_plan_desc *desc, int device, qx_plan *out) {
         if (d.ldc == 0) d.ldc = d.N;
         if (d.lda < d.K || d.ldb < d.N || d.ldc < d.N)
             return fail(QX_ERR_INVALID_ARG, "leading dimension shorter than the row");
+        if ((d.flags & QX_FLAG_FUSED_CONVERT) && !gemm_rows_aligned(d))
+            return fail(QX_ERR_UNSUPPORTED,
+                        "the fused path needs 16-byte aligned rows (lda, ldb multiples of %d)",
+                        d.in_dtype == QX_I32 ? 4 : 8);
     }
     qx_plan_s tmp;
     int s_shift = 0, max_keys = 0;
@@ -1192,10 +1249,25 @@ static qx_status execute(qx_plan p, qx_op op, qx_dtype want, const void *a, cons
     if (op == QX_OP_GEMM && (d.M == 0 || d.N == 0)) return QX_OK;
     if (!out) return fail(QX_ERR_INVALID_ARG, "null output");
     if (!aligned16(out)) return fail(QX_ERR_UNSUPPORTED, "output must be 16-byte aligned");
+    if (op == QX_OP_GEMM && p->fused && d.K > 0) {
+        if (!a || !b) return fail(QX_ERR_INVALID_ARG, "null operand");
+        if (!aligned16(a) || !aligned16(b))
+            return fail(QX_ERR_UNSUPPORTED, "operand base pointers must be 16-byte aligned");
+        MmaArgs m = p->fmma;
+        m.raw_a = a;
+        m.raw_b = b;
+        m.out = out;
+        QX_CUDA(fused_gemm_launch(p->scheme[0].n.limbs, p->scheme[0].m.limbs, d.in_dtype == QX_I32,
+                                  p->fused_packed, m, p->fgrid, st),
+                "fused GEMM launch");
+        return QX_OK;
+    }
     qx_status s = pack(p, a, b, c, st);
     if (s != QX_OK) return s;
     return run_packed(p, out, st);
 }
+
+int qx_plan_fused(qx_plan p) { return p ? (p->fused ? 1 : 0) : -1; }
 
 qx_status qx_gemm_i16_i32(qx_plan p, const int16_t *A, const int16_t *B, int32_t *C,
                           qx_stream stream) {

@@ -1,0 +1,597 @@
+// qx_fused.cu -- the tiled limb GEMM with the limb conversion fused into the
+// kernel: the integer operands are read straight from the caller's int16 or
+// int32 matrices and split into FP16 digits in shared memory, so the call is
+// one launch with no packed planes in HBM (paper: Methodology, persistent
+// executors and operand-range contracts that decide packing at runtime;
+// Table 1 GEMM rows).
+//
+// The arithmetic is the limb GEMM's (qx_mma.cu): the same balanced digits, the
+// same FP32 chunks bounded by 2^24, the same drain and wrapping int32
+// recombination, the same tile geometry and shared-memory layout (K-major,
+// 128-byte swizzled rows), so both kernels give the same bits.  Only the
+// producer differs: instead of TMA loads of packed planes, eight converter
+// warps copy raw integer tiles into a small ring of their own with cp.async
+// (16-byte copies, zero-filled past the matrix edges, `RD - 1` k-blocks
+// ahead), split every element into its digits and store the digit rows into
+// the stage ring in the swizzled layout the MMA descriptors expect.  Each
+// converter thread copies exactly the raw words it later converts, so its own
+// cp.async groups are the only thing it waits for.
+//
+// Roles (288 threads):
+//   warp 0      TMEM owner and MMA issuer (one thread), as in qx_mma.cu
+//   warps 1..8  converters during the main loop, epilogue at chunk ends
+//               (the tiles of a small problem fit one wave, so a CTA has no
+//               next tile whose conversion the epilogue would hold up).
+// Converter work per k-block: threads 0..127 transpose B (K x N, row-major)
+// into the M-side tile, one 8 k x 8 n block each; threads 128..255 split
+// MR rows x 64 k of A into the N-side tile, 8 consecutive k per item.
+#include <cuda.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include "qx_device.cuh"
+#include "qx_internal.h"
+#include "qx_tile.cuh"
+
+namespace qx {
+
+template <typename T, int NA, int NB>
+struct FusedCfg {
+    using L = TileCfg<NA, NB, kKindExact>;
+    static constexpr int THREADS = 288;
+    static constexpr int CONV_WARPS = 8;
+    static constexpr int W = int(sizeof(T)) / 2;      // 16-byte words per 8 elements
+    static constexpr int N_ITEMS = L::MR / 16;        // N-side rows per converter thread
+    // raw ring: M side [8 rows][W][128 threads] then N side [N_ITEMS][W][128], 16 B each
+    static constexpr int RAW_M = 8 * W * 128 * 16;
+    static constexpr int RAW = RAW_M + N_ITEMS * W * 128 * 16;
+    static constexpr int BUDGET = 232448 - 1024 - 256;   // opt-in shared memory per CTA
+    static constexpr int RD = (BUDGET - 2 * RAW) / L::STAGE >= 2 ? 2 : 1;
+    static constexpr int SD_FIT = (BUDGET - RD * RAW) / L::STAGE;
+    static constexpr int STAGES = SD_FIT > 4 ? 4 : SD_FIT;
+    static constexpr int SMEM = STAGES * L::STAGE + RD * RAW + 256 + 1024;
+    static_assert(STAGES >= 2, "stage ring too small");
+    static_assert(SMEM <= 232448, "shared memory over the per-CTA limit");
+};
+
+// 16-byte asynchronous copy global -> shared; bytes past `src_bytes` (0..16)
+// are filled with zeros and not read.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+__device__ __forceinline__ uint32_t word_of(const uint4 &w, int i) {
+    return i == 0 ? w.x : i == 1 ? w.y : i == 2 ? w.z : w.w;
+}
+
+// Element e (0..7, a compile-time constant after unrolling) of a group.
+template <typename T>
+__device__ __forceinline__ int32_t elem(const uint4 (&w)[sizeof(T) / 2], int e) {
+    if constexpr (sizeof(T) == 2) {
+        const uint32_t u = word_of(w[0], e >> 1);
+        return (e & 1) ? int32_t(u) >> 16 : int32_t(u << 16) >> 16;
+    } else {
+        return int32_t(word_of(w[e >> 2], e & 3));
+    }
+}
+
+// One FP16 value of an integer digit |d| <= 2048: d + 1.5 * 2^23 is exact in
+// binary32, and so is subtracting the constant back; FP16 holds d exactly.
+__device__ __forceinline__ float digit_float(int32_t d) {
+    return __int_as_float(0x4B400000 + d) - 12582912.0f;
+}
+
+// The NL digits of 8 values as NL rows of 8 FP16 values (one uint4 each).
+template <int NL>
+__device__ __forceinline__ void digits8(const int32_t (&v)[8], int shift, uint4 (&out)[NL]) {
+    uint32_t h[NL][4];
+#pragma unroll
+    for (int e = 0; e < 8; e += 2) {
+        int32_t d0[NL], d1[NL];
+        split_digits<NL>(v[e], shift, d0);
+        split_digits<NL>(v[e + 1], shift, d1);
+#pragma unroll
+        for (int i = 0; i < NL; ++i) {
+            const __half2 p = __floats2half2_rn(digit_float(d0[i]), digit_float(d1[i]));
+            h[i][e / 2] = *reinterpret_cast<const uint32_t *>(&p);
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < NL; ++i) out[i] = make_uint4(h[i][0], h[i][1], h[i][2], h[i][3]);
+}
+
+__device__ __forceinline__ void range_test(int32_t v, int64_t lo, int64_t hi, int *err) {
+    if (v < lo || v > hi) atomicCAS(err, 0, kErrContract);
+}
+
+// ---- packed conversion: two int16 values per 32-bit word, FP16 pairs out.
+// Every step is exact.  An FP16 value with bits 0x6400 | u (u < 1024) is
+// 1024 + u, so masking bits of the integer into that pattern and subtracting
+// the bias in FP16 gives small integers directly.  A value x (int16) is
+// written as x = 512 h + l with l = x mod 512 in [0, 512) and h = x >> 9 in
+// [-64, 64): l from the low 9 bits, h from bits 9..15 in offset binary.
+__device__ __forceinline__ __half2 as_h2(uint32_t u) { return *reinterpret_cast<const __half2 *>(&u); }
+__device__ __forceinline__ uint32_t as_u32(__half2 h) { return *reinterpret_cast<const uint32_t *>(&h); }
+
+struct PackedConsts {
+    __half2 c1024, c1088, c512;   // biases and the weight of h
+    __half2 lo_bias, inv, neg_inv, up;   // two-digit split of shift s
+    uint32_t lo_mask, lo_xor;
+    __device__ __forceinline__ void init(int s) {
+        c1024 = __float2half2_rn(1024.0f);
+        c1088 = __float2half2_rn(1088.0f);
+        c512 = __float2half2_rn(512.0f);
+        if (s > 0) {
+            lo_mask = ((1u << s) - 1u) * 0x00010001u;
+            lo_xor = (0x6400u | (1u << (s - 1))) * 0x00010001u;
+            lo_bias = __float2half2_rn(float(1024 + (1 << (s - 1))));
+            inv = __float2half2_rn(__int_as_float((127 - s) << 23));       // 2^-s
+            neg_inv = __float2half2_rn(-__int_as_float((127 - s) << 23));
+            up = __float2half2_rn(float(1 << (9 - s)));                     // 2^(9-s)
+        }
+    }
+};
+
+__device__ __forceinline__ void pk_split9(uint32_t w, const PackedConsts &c, __half2 &l, __half2 &h) {
+    l = __hsub2(as_h2((w & 0x01FF01FFu) | 0x64006400u), c.c1024);
+    h = __hsub2(as_h2(((w >> 9) & 0x007F007Fu) ^ 0x64406440u), c.c1088);
+}
+
+// A whole operand (|x| <= 2048): x = 512 h + l, one FMA, exact.
+__device__ __forceinline__ uint32_t pk_whole(uint32_t w, const PackedConsts &c) {
+    __half2 l, h;
+    pk_split9(w, c, l, h);
+    return as_u32(__hfma2(h, c.c512, l));
+}
+
+// Two balanced digits of shift s <= 9: lo = ((x + 2^(s-1)) mod 2^s) - 2^(s-1)
+// from the low s bits, hi = (x - lo) / 2^s = h 2^(9-s) + (l - lo) / 2^s.
+__device__ __forceinline__ void pk_two(uint32_t w, const PackedConsts &c, uint32_t &lo_out, uint32_t &hi_out) {
+    const __half2 lo = __hsub2(as_h2((w & c.lo_mask) ^ c.lo_xor), c.lo_bias);
+    __half2 l, h;
+    pk_split9(w, c, l, h);
+    const __half2 m = __hfma2(l, c.inv, __hmul2(lo, c.neg_inv));
+    lo_out = as_u32(lo);
+    hi_out = as_u32(__hfma2(h, c.up, m));
+}
+
+// The NL digit words of one packed pair.
+template <int NL>
+__device__ __forceinline__ void pk_digits(uint32_t w, const PackedConsts &c, uint32_t (&d)[NL]) {
+    static_assert(NL == 1 || NL == 2, "packed digits: one or two limbs");
+    if constexpr (NL == 1) d[0] = pk_whole(w, c);
+    else pk_two(w, c, d[0], d[1]);
+}
+
+// Word j (0..3) of a group of 8 elements as a packed int16 pair; int32
+// elements are narrowed (their declared range fits int16).
+template <typename T>
+__device__ __forceinline__ uint32_t pair_word(const uint4 (&w)[sizeof(T) / 2], int j) {
+    if constexpr (sizeof(T) == 2) {
+        return word_of(w[0], j);
+    } else {
+        return __byte_perm(word_of(w[j >> 1], (j & 1) * 2), word_of(w[j >> 1], (j & 1) * 2 + 1), 0x5410);
+    }
+}
+
+// Packed pair (element e of group ra, element e of group rb).
+template <typename T>
+__device__ __forceinline__ uint32_t column_pair(const uint4 (&ra)[sizeof(T) / 2], const uint4 (&rb)[sizeof(T) / 2],
+                                                int e) {
+    if constexpr (sizeof(T) == 2) {
+        return __byte_perm(word_of(ra[0], e >> 1), word_of(rb[0], e >> 1), (e & 1) ? 0x7632 : 0x5410);
+    } else {
+        return __byte_perm(word_of(ra[e >> 2], e & 3), word_of(rb[e >> 2], e & 3), 0x5410);
+    }
+}
+
+template <typename T, int NA, int NB, bool PK>
+__global__ void __launch_bounds__(288, 1) fused_gemm_kernel(const __grid_constant__ MmaArgs a) {
+    using F = FusedCfg<T, NA, NB>;
+    using L = typename F::L;
+    constexpr int W = F::W;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *raw_ring = smem + F::STAGES * L::STAGE;
+    uint64_t *full = reinterpret_cast<uint64_t *>(raw_ring + F::RD * F::RAW);
+    uint64_t *empty = full + F::STAGES;
+    uint64_t *acc_full = empty + F::STAGES;
+    uint64_t *acc_empty = acc_full + 2;
+    uint64_t *tail = acc_empty + 2;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(tail + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int ntiles = a.tiles_m * a.tiles_n;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < F::STAGES; ++s) {
+            mbar_init(&full[s], F::CONV_WARPS);   // one arrival per converter warp
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], F::CONV_WARPS);
+        }
+        mbar_init(tail, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(tmem_slot, L::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    // the operands may come from the kernel launched just before this one
+    pdl_wait();
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // -------------------------------------------------- MMA issuer
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t acc_it = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+                for (int kb0 = 0; kb0 < a.kblocks; kb0 += a.chunk_kb) {
+                    const int kb1 = min(kb0 + a.chunk_kb, a.kblocks);
+                    const uint32_t buf = L::NBUF == 2 ? (acc_it & 1u) : 0u;
+                    const uint32_t apar = L::NBUF == 2 ? ((acc_it >> 1) & 1u) : (acc_it & 1u);
+                    if (!mbar_wait(&acc_empty[buf], apar ^ 1, abort_flag, a.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t d0 = tmem_base + buf * L::ACC_COLS;
+                    for (int kb = kb0; kb < kb1; ++kb) {
+                        if (!mbar_wait(&full[stage], phase, abort_flag, a.err)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t sbase = smem_addr(smem + stage * L::STAGE);
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk) {
+                            const uint64_t bdesc = make_sdesc(sbase + NB * L::M_TILE + kk * 32);
+                            const uint32_t acc = (kb > kb0 || kk > 0) ? 1u : 0u;
+#pragma unroll
+                            for (int j = 0; j < NB; ++j)
+                                mma_f16(d0 + j * L::UN, make_sdesc(sbase + j * L::M_TILE + kk * 32), bdesc,
+                                        L::IDESC, acc);
+                        }
+                        tc_commit(&empty[stage]);
+                        if (++stage == F::STAGES) {
+                            stage = 0;
+                            phase ^= 1;
+                        }
+                    }
+                    if (!ok) break;
+                    tc_commit(&acc_full[buf]);
+                    ++acc_it;
+                }
+            }
+            if (!ok) {
+                // MMAs already issued must finish before TMEM is released.
+                tc_commit(tail);
+                mbar_wait_drain(tail, 0);
+            }
+        }
+    } else {
+        // --------------------------------------- converters, then epilogue
+        const int ct = threadIdx.x - 32;          // 0 .. 255
+        const bool mside = ct < 128;
+        const int kg = ct & 7;                    // 8-wide k group of the k-block
+        const int grp = (ct & 127) >> 3;          // 0 .. 15
+        const int q = warp & 3;                   // TMEM lane quarter this warp may read
+        const int hh = (warp - 1) >> 2;           // which half of the N-side rows
+        const T *A = static_cast<const T *>(a.raw_a);
+        const T *B = static_cast<const T *>(a.raw_b);
+        const bool chk = a.chk != 0;
+        int stage = 0;
+        uint32_t phase = 0;
+        uint32_t acc_it = 0;
+        bool ok = true;
+        // this thread's raw words: M side, k row kg*8 + r of the 8 x 8 block
+        // at columns grp*8 ..; N side, A row grp + 16 r at k kg*8 ..
+        const uint32_t raw_base = smem_addr(raw_ring) + (mside ? 0u : uint32_t(F::RAW_M)) +
+                                  uint32_t(ct & 127) * 16u;
+        auto raw_off = [](int r, int i) { return uint32_t((r * W + i) * 128 * 16); };
+
+        auto issue = [&](int tm, int tn, int kb) {
+            const uint32_t dst = raw_base + uint32_t(kb % F::RD) * F::RAW;
+            const int k0 = kb * kBK + kg * 8;
+            if (mside) {
+                const int n = tm * kBM + grp * 8;
+                const int valid_n = max(0, min(8, a.m_extent - n));
+#pragma unroll
+                for (int r = 0; r < 8; ++r) {
+                    const int k = k0 + r;
+                    const int valid = k < a.K ? valid_n : 0;
+                    const T *src = valid > 0 ? B + int64_t(k) * a.ldb + n : B;
+#pragma unroll
+                    for (int i = 0; i < W; ++i) {
+                        const int bytes = min(max(valid * int(sizeof(T)) - 16 * i, 0), 16);
+                        cp_async16(dst + raw_off(r, i), bytes > 0 ? src + 8 / W * i : B, bytes);
+                    }
+                }
+            } else {
+                const int valid_k = max(0, min(8, a.K - k0));
+#pragma unroll
+                for (int r = 0; r < F::N_ITEMS; ++r) {
+                    const int row = tn * L::MR + grp + 16 * r;
+                    const int valid = row < a.n_extent ? valid_k : 0;
+                    const T *src = valid > 0 ? A + int64_t(row) * a.lda + k0 : A;
+#pragma unroll
+                    for (int i = 0; i < W; ++i) {
+                        const int bytes = min(max(valid * int(sizeof(T)) - 16 * i, 0), 16);
+                        cp_async16(dst + raw_off(r, i), bytes > 0 ? src + 8 / W * i : A, bytes);
+                    }
+                }
+            }
+        };
+        auto read_raw = [&](int kb, int r, uint4 (&w)[W]) {
+            const uint32_t src = raw_base + uint32_t(kb % F::RD) * F::RAW + raw_off(r, 0);
+#pragma unroll
+            for (int i = 0; i < W; ++i) {
+                uint4 v;
+                asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                             : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                             : "r"(src + uint32_t(i * 128 * 16)));
+                w[i] = v;
+            }
+        };
+        PackedConsts pkc;
+        if constexpr (PK) pkc.init(mside ? (NB == 2 ? a.shift_m : 0) : (NA == 2 ? a.shift_n : 0));
+        auto convert = [&](int tm, int tn, int kb, uint8_t *st) {
+            const int k0 = kb * kBK + kg * 8;
+            if (mside) {
+                uint4 raw[8][W];
+#pragma unroll
+                for (int r = 0; r < 8; ++r) read_raw(kb, r, raw[r]);
+                const int n = tm * kBM + grp * 8;
+                if (chk) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+#pragma unroll
+                        for (int r = 0; r < 8; ++r)
+                            if (k0 + r < a.K && n + e < a.m_extent)
+                                range_test(elem<T>(raw[r], e), a.lo_b, a.hi_b, a.err);
+                }
+                // column e of the 8 x 8 block -> M-side row grp*8 + e, chunk kg
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    uint4 d[NB];
+                    if constexpr (PK) {
+                        uint32_t dw[4][NB];
+#pragma unroll
+                        for (int p = 0; p < 4; ++p) pk_digits<NB>(column_pair<T>(raw[2 * p], raw[2 * p + 1], e), pkc, dw[p]);
+#pragma unroll
+                        for (int j = 0; j < NB; ++j) d[j] = make_uint4(dw[0][j], dw[1][j], dw[2][j], dw[3][j]);
+                    } else {
+                        int32_t v[8];
+#pragma unroll
+                        for (int r = 0; r < 8; ++r) v[r] = elem<T>(raw[r], e);
+                        digits8<NB>(v, a.shift_m, d);
+                    }
+                    const int row = grp * 8 + e;
+#pragma unroll
+                    for (int j = 0; j < NB; ++j)
+                        *reinterpret_cast<uint4 *>(st + j * L::M_TILE + row * 128 + ((kg ^ (row & 7)) << 4)) = d[j];
+                }
+            } else {
+#pragma unroll
+                for (int r = 0; r < F::N_ITEMS; ++r) {
+                    uint4 raw[W];
+                    read_raw(kb, r, raw);
+                    const int row = grp + 16 * r;
+                    if (chk && tn * L::MR + row < a.n_extent) {
+#pragma unroll
+                        for (int e = 0; e < 8; ++e)
+                            if (k0 + e < a.K) range_test(elem<T>(raw, e), a.lo_a, a.hi_a, a.err);
+                    }
+                    uint4 d[NA];
+                    if constexpr (PK) {
+                        uint32_t dw[4][NA];
+#pragma unroll
+                        for (int p = 0; p < 4; ++p) pk_digits<NA>(pair_word<T>(raw, p), pkc, dw[p]);
+#pragma unroll
+                        for (int i = 0; i < NA; ++i) d[i] = make_uint4(dw[0][i], dw[1][i], dw[2][i], dw[3][i]);
+                    } else {
+                        int32_t v[8];
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) v[e] = elem<T>(raw, e);
+                        digits8<NA>(v, a.shift_n, d);
+                    }
+#pragma unroll
+                    for (int i = 0; i < NA; ++i)
+                        *reinterpret_cast<uint4 *>(st + NB * L::M_TILE + i * L::MR * 128 + row * 128 +
+                                                   ((kg ^ (row & 7)) << 4)) = d[i];
+                }
+            }
+        };
+        // Drain one chunk straight into C: no running sums stay in registers
+        // while the warp converts.  The first chunk of a tile stores, later
+        // chunks add to what this thread stored before (wrapping int32), and
+        // the last applies the optional ReLU-requantize.
+        const int nchunks = (a.kblocks + a.chunk_kb - 1) / a.chunk_kb;
+        auto drain = [&](int tm, int tn, int c) -> bool {
+            const uint32_t buf = L::NBUF == 2 ? (acc_it & 1u) : 0u;
+            const uint32_t apar = L::NBUF == 2 ? ((acc_it >> 1) & 1u) : (acc_it & 1u);
+            if (!mbar_wait(&acc_full[buf], apar, abort_flag, a.err)) return false;
+            tc_fence_after();
+            const uint32_t tb = tmem_base + (uint32_t(q * 32) << 16) + buf * L::ACC_COLS + hh * L::RPT;
+            const int mrow = tm * kBM + q * 32 + lane;
+            const bool lane_ok = mrow < a.m_extent;
+            const int nrow0 = tn * L::MR + hh * L::RPT;
+            const int rows_left = a.n_extent - nrow0;
+            uint32_t *o = static_cast<uint32_t *>(a.out) + mrow + int64_t(nrow0) * a.out_row_stride;
+            const bool first = c == 0, last = c == nchunks - 1;
+#pragma unroll
+            for (int pg = 0; pg < L::RPT / 32; ++pg) {
+                if (pg * 32 >= rows_left) continue;
+                uint32_t sum[32];
+#pragma unroll
+                for (int x = 0; x < 32; ++x) sum[x] = 0u;
+#pragma unroll
+                for (int j = 0; j < NB; ++j) {
+#pragma unroll
+                    for (int i = 0; i < NA; ++i) {
+                        const int sh = i * a.shift_n + j * a.shift_m;
+                        uint32_t v[32];
+                        tmem_ld32(tb + j * L::UN + i * L::MR + pg * 32, v);
+                        tmem_wait_ld(v);
+#pragma unroll
+                        for (int x = 0; x < 32; ++x)
+                            sum[x] += uint32_t(__float2int_rn(__uint_as_float(v[x]))) << sh;
+                    }
+                }
+                if (!first) {
+                    // every earlier partial is loaded before any store, so
+                    // the 32 loads are in flight together
+                    uint32_t prev[32];
+#pragma unroll
+                    for (int x = 0; x < 32; ++x) {
+                        const int r = pg * 32 + x;
+                        prev[x] = (lane_ok && r < rows_left) ? o[int64_t(r) * a.out_row_stride] : 0u;
+                    }
+#pragma unroll
+                    for (int x = 0; x < 32; ++x) sum[x] += prev[x];
+                }
+#pragma unroll
+                for (int x = 0; x < 32; ++x) {
+                    const int r = pg * 32 + x;
+                    if (!lane_ok || r >= rows_left) continue;
+                    uint32_t val = sum[x];
+                    if (last && a.rq_on) val = uint32_t(min(max(int32_t(val), 0) >> a.rq_shift, a.rq_hi));
+                    o[int64_t(r) * a.out_row_stride] = val;
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acc_empty[buf]);
+            ++acc_it;
+            return true;
+        };
+
+        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+            int tm, tn;
+            tile_coords(t, a, tm, tn);
+            for (int p = 0; p < F::RD - 1; ++p) {
+                if (p < a.kblocks) issue(tm, tn, p);
+                cp_async_commit();
+            }
+            // With two accumulator sets, chunk c is drained after chunk c + 1
+            // has been converted, so the tensor cores never wait for a drain;
+            // with one set, each chunk is drained as soon as it is converted.
+            for (int kb = 0; ok && kb < a.kblocks; ++kb) {
+                if (kb + F::RD - 1 < a.kblocks) issue(tm, tn, kb + F::RD - 1);
+                cp_async_commit();
+                cp_async_wait<F::RD - 1>();            // this thread's copies of k-block kb
+                if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, a.err)) {
+                    ok = false;
+                    break;
+                }
+                convert(tm, tn, kb, smem + stage * L::STAGE);
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&full[stage]);
+                if (++stage == F::STAGES) {
+                    stage = 0;
+                    phase ^= 1;
+                }
+                const bool chunk_end = (kb + 1) % a.chunk_kb == 0 || kb + 1 == a.kblocks;
+                const int c = kb / a.chunk_kb;
+                if (chunk_end && L::NBUF == 1) ok = drain(tm, tn, c);
+                else if (chunk_end && c >= 1) ok = drain(tm, tn, c - 1);
+            }
+            if (ok && L::NBUF == 2) ok = drain(tm, tn, nchunks - 1);   // the tile's last chunk
+        }
+        cp_async_wait<0>();   // no copy into the raw ring outlives the CTA
+        if (ok && ct == 0) {
+            // Every stage must be released by the MMA before the CTA exits,
+            // so that no commit lands on the barriers of a later CTA.
+            for (int i = 0; i < F::STAGES; ++i) {
+                if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, a.err)) break;
+                if (++stage == F::STAGES) {
+                    stage = 0;
+                    phase ^= 1;
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, L::TMEM_COLS);
+    }
+}
+
+// ------------------------------------------------------------------- host
+template <typename T, int NA, int NB, bool PK>
+static cudaError_t fused_prepare_t() {
+    return cudaFuncSetAttribute(fused_gemm_kernel<T, NA, NB, PK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                FusedCfg<T, NA, NB>::SMEM);
+}
+
+template <typename T, int NA, int NB, bool PK>
+static cudaError_t fused_launch_t(const MmaArgs &a, int grid, cudaStream_t stream) {
+    using F = FusedCfg<T, NA, NB>;
+    return launch_pdl(fused_gemm_kernel<T, NA, NB, PK>, grid, F::THREADS, F::SMEM, stream, a);
+}
+
+// Packed conversion exists for one or two limbs per side.
+template <int NA, int NB>
+static cudaError_t fused_prepare_n(bool i32, bool pk) {
+    if constexpr (NA <= 2 && NB <= 2) {
+        if (pk) return i32 ? fused_prepare_t<int32_t, NA, NB, true>() : fused_prepare_t<int16_t, NA, NB, true>();
+    }
+    return i32 ? fused_prepare_t<int32_t, NA, NB, false>() : fused_prepare_t<int16_t, NA, NB, false>();
+}
+
+template <int NA, int NB>
+static cudaError_t fused_launch_n(bool i32, bool pk, const MmaArgs &a, int grid, cudaStream_t stream) {
+    if constexpr (NA <= 2 && NB <= 2) {
+        if (pk)
+            return i32 ? fused_launch_t<int32_t, NA, NB, true>(a, grid, stream)
+                       : fused_launch_t<int16_t, NA, NB, true>(a, grid, stream);
+    }
+    return i32 ? fused_launch_t<int32_t, NA, NB, false>(a, grid, stream)
+               : fused_launch_t<int16_t, NA, NB, false>(a, grid, stream);
+}
+
+#define QX_FUSED_DISPATCH(FN, ...)                                         \
+    switch (na * 10 + nb) {                                                \
+        case 11: return FN<1, 1>(__VA_ARGS__);                             \
+        case 21: return FN<2, 1>(__VA_ARGS__);                             \
+        case 31: return FN<3, 1>(__VA_ARGS__);                             \
+        case 41: return FN<4, 1>(__VA_ARGS__);                             \
+        case 12: return FN<1, 2>(__VA_ARGS__);                             \
+        case 22: return FN<2, 2>(__VA_ARGS__);                             \
+        case 42: return FN<4, 2>(__VA_ARGS__);                             \
+        default: return cudaErrorInvalidValue;                             \
+    }
+
+// Whether the packed conversion applies: every operand value fits int16 and
+// each side has one limb (|x| <= 2048) or two limbs of at most 9 bits.
+bool fused_gemm_packed_ok(int na, int shift_n, int nb, int shift_m, bool values_fit_int16) {
+    return values_fit_int16 && na <= 2 && nb <= 2 && (na == 1 || shift_n <= 9) && (nb == 1 || shift_m <= 9);
+}
+
+cudaError_t fused_gemm_prepare(int na, int nb, bool i32, bool pk) { QX_FUSED_DISPATCH(fused_prepare_n, i32, pk) }
+
+cudaError_t fused_gemm_launch(int na, int nb, bool i32, bool pk, const MmaArgs &a, int grid, cudaStream_t stream) {
+    QX_FUSED_DISPATCH(fused_launch_n, i32, pk, a, grid, stream)
+}
+
+}  // namespace qx

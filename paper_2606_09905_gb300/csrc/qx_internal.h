@@ -62,11 +62,19 @@ struct MmaArgs {
     int kblocks;              // ceil(K / kBK)
     int chunk_kb;             // k-blocks per FP32 accumulation chunk
     int tiles_m, tiles_n, group_n;
+    int mr;                   // N-side rows per limb of the tile (128 or 64)
     int shift_n, shift_m;     // digit widths of the N-side / M-side limbs
     // conv geometry (modes 1 and 2)
     int c_blocks, S, Q, PQ, stride, pad, k_out;
     // output = min(max(acc, 0) >> rq_shift, rq_hi) when rq_on (integer kinds)
     int rq_on, rq_shift, rq_hi;
+    // fused conversion (GEMM only): raw integer operands, set per call
+    const void *raw_a;        // A, M x K row-major (N side)
+    const void *raw_b;        // B, K x N row-major (M side)
+    int64_t lda, ldb;         // row strides in elements
+    int K;
+    int chk;                  // compare every element with its declared range
+    int64_t lo_a, hi_a, lo_b, hi_b;
 };
 
 // Kernel arguments of the fused attention core.

@@ -37,63 +37,13 @@
 
 #include "qx_device.cuh"
 #include "qx_internal.h"
+#include "qx_tile.cuh"
 
 namespace qx {
 
-template <int NA, int NB, int KIND>
-struct TileCfg {
-    static constexpr bool TF = KIND == kKindTf32x3;
-    static constexpr int MR = NA <= 2 ? 128 : 64;   // N-side rows per limb
-    static constexpr int UN = NA * MR;              // MMA N
-    static constexpr int M_TILE = kBM * 128;        // bytes of one M-side limb tile
-    static constexpr int N_TILE = UN * 128;         // bytes of the stacked N-side tile
-    static constexpr int STAGE = NB * M_TILE + N_TILE;
-    static constexpr int STAGES_FIT = (200 * 1024) / STAGE;
-    static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
-    // TMEM columns per accumulator set: every M-side limb has its own for the
-    // exact kind; the TF32 kind sums all products into one.
-    static constexpr int ACC_COLS = TF ? UN : NB * UN;
-    static constexpr int NBUF = ACC_COLS <= 256 ? 2 : 1;
-    static constexpr int TMEM_NEED = ACC_COLS * NBUF;
-    static constexpr int TMEM_COLS = TMEM_NEED <= 32    ? 32
-                                     : TMEM_NEED <= 64  ? 64
-                                     : TMEM_NEED <= 128 ? 128
-                                     : TMEM_NEED <= 256 ? 256
-                                                        : 512;
-    static constexpr int RPT = MR / 2;              // N-side rows per epilogue thread
-    static constexpr uint32_t AB_TYPE = TF ? 2u : 0u;
-    static constexpr uint32_t IDESC = make_idesc(kBM, UN, AB_TYPE);
-    static constexpr uint32_t IDESC_FIRST = make_idesc(kBM, MR, AB_TYPE);  // first N-side limb only
-    static constexpr int BK_ELEMS = TF ? kBK32 : kBK;                     // K per 128-byte row
-    static constexpr int BAR_BYTES = 256;
-    static constexpr int SMEM = STAGES * STAGE + BAR_BYTES + 1024;
-    // warp 0: M-side TMA producer; warp 1: TMEM + MMA issue; warps 2-9:
-    // epilogue; warp 10: N-side TMA producer.  One thread needs a few hundred
-    // cycles to issue a TMA load, so two producer threads keep a k-block's
-    // loads within its MMA time.
-    static constexpr int THREADS = 352;
-    static constexpr int N_PRODUCER_WARP = 10;
-    static_assert(UN % 16 == 0 && UN >= 16 && UN <= 256, "MMA N out of range");
-    static_assert(TMEM_NEED <= 512, "accumulators exceed tensor memory");
-    static_assert(RPT % 32 == 0, "epilogue works in 32-column TMEM loads");
-    static_assert(!TF || (NA == 2 && NB == 2), "TF32x3 stacks big/small on both sides");
-};
-
-// Tile order: groups of `group_n` N-side tiles, M-side tiles inside a group,
-// so the CTAs resident at one time share operand tiles through L2.
-__device__ __forceinline__ void tile_coords(int t, const MmaArgs &a, int &tm, int &tn) {
-    const int per_group = a.group_n * a.tiles_m;
-    const int g = t / per_group;
-    const int first = g * a.group_n;
-    const int gs = min(a.group_n, a.tiles_n - first);
-    const int r = t - g * per_group;
-    tn = first + r % gs;
-    tm = r / gs;
-}
-
-template <int NA, int NB, int KIND>
+template <int NA, int NB, int KIND, int MR_>
 __global__ void __launch_bounds__(352, 1) limb_gemm_kernel(const __grid_constant__ MmaArgs a) {
-    using T = TileCfg<NA, NB, KIND>;
+    using T = TileCfg<NA, NB, KIND, MR_>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -338,26 +288,8 @@ __global__ void __launch_bounds__(352, 1) limb_gemm_kernel(const __grid_constant
                                 (__uint_as_float(v0[x]) + __uint_as_float(v1[x])));
                     }
                 } else {
-                    // 32-row chunks wholly past the N-side extent hold nothing to keep
-                    const int rows_left = a.n_extent - (tn * T::MR + hh * T::RPT);
-#pragma unroll
-                    for (int j = 0; j < NB; ++j) {
-#pragma unroll
-                        for (int i = 0; i < NA; ++i) {
-                            const int sh = i * a.shift_n + j * a.shift_m;
-#pragma unroll
-                            for (int p = 0; p < T::RPT / 32; ++p) {
-                                if (p * 32 >= rows_left) continue;
-                                uint32_t v[32];
-                                tmem_ld32(tb + j * T::UN + i * T::MR + p * 32, v);
-                                tmem_wait_ld(v);
-#pragma unroll
-                                for (int x = 0; x < 32; ++x)
-                                    acc[p * 32 + x] +=
-                                        uint32_t(__float2int_rn(__uint_as_float(v[x]))) << sh;
-                            }
-                        }
-                    }
+                    drain_exact<NA, NB, MR_>(tb, a.n_extent - (tn * T::MR + hh * T::RPT), a.shift_n,
+                                        a.shift_m, acc);
                 }
                 tc_fence_before();
                 __syncwarp();
@@ -365,27 +297,7 @@ __global__ void __launch_bounds__(352, 1) limb_gemm_kernel(const __grid_constant
                 ++acc_it;
             }
             if (!ok) break;
-            const int mrow = tm * kBM + q * 32 + lane;
-            const bool lane_ok = mrow < a.m_extent;
-            int64_t lane_off = mrow;
-            if (a.mode != 0) {   // conv: pixel mrow of image img, NCHW output
-                const int img = mrow / a.PQ;
-                lane_off = int64_t(img) * a.k_out * a.PQ + (mrow - img * a.PQ);
-            }
-            if constexpr (!T::TF) {
-                if (a.rq_on) {   // ReLU, requantizing shift, clamp
-#pragma unroll
-                    for (int r = 0; r < T::RPT; ++r)
-                        acc[r] = uint32_t(min(max(int32_t(acc[r]), 0) >> a.rq_shift, a.rq_hi));
-                }
-            }
-            const int nrow0 = tn * T::MR + hh * T::RPT;
-            // both output types are 32-bit: store the raw words
-            uint32_t *o = static_cast<uint32_t *>(a.out) + lane_off + int64_t(nrow0) * a.out_row_stride;
-#pragma unroll
-            for (int r = 0; r < T::RPT; ++r) {
-                if (lane_ok && nrow0 + r < a.n_extent) o[int64_t(r) * a.out_row_stride] = acc[r];
-            }
+            store_tile<NA, NB, KIND, MR_>(a, tm, tn, q, hh, lane, acc);
         }
     }
 
@@ -398,20 +310,32 @@ __global__ void __launch_bounds__(352, 1) limb_gemm_kernel(const __grid_constant
 }
 
 // ------------------------------------------------------------------- host
-template <int NA, int NB, int KIND = kKindExact>
+template <int NA, int NB, int KIND = kKindExact, int MR_ = TileCfg<NA, NB, KIND>::MR>
 static cudaError_t prepare_t() {
-    return cudaFuncSetAttribute(limb_gemm_kernel<NA, NB, KIND>,
+    return cudaFuncSetAttribute(limb_gemm_kernel<NA, NB, KIND, MR_>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                TileCfg<NA, NB, KIND>::SMEM);
+                                TileCfg<NA, NB, KIND, MR_>::SMEM);
 }
 
-template <int NA, int NB, int KIND = kKindExact>
+template <int NA, int NB, int KIND = kKindExact, int MR_ = TileCfg<NA, NB, KIND>::MR>
 static cudaError_t launch_t(const MmaArgs &a, int grid, cudaStream_t stream) {
-    using T = TileCfg<NA, NB, KIND>;
-    return launch_pdl(limb_gemm_kernel<NA, NB, KIND>, grid, T::THREADS, T::SMEM, stream, a);
+    using T = TileCfg<NA, NB, KIND, MR_>;
+    return launch_pdl(limb_gemm_kernel<NA, NB, KIND, MR_>, grid, T::THREADS, T::SMEM, stream, a);
 }
 
+// Instances: every limb pair at the default rows per limb, and one or two
+// limbs per side at 64 rows (small problems).
 #define QX_LIMB_DISPATCH(FN, ...)                                          \
+    if (mr == 64 && na <= 2) {                                             \
+        switch (na * 10 + nb) {                                            \
+            case 11: return FN<1, 1, kKindExact, 64>(__VA_ARGS__);         \
+            case 21: return FN<2, 1, kKindExact, 64>(__VA_ARGS__);         \
+            case 12: return FN<1, 2, kKindExact, 64>(__VA_ARGS__);         \
+            case 22: return FN<2, 2, kKindExact, 64>(__VA_ARGS__);         \
+            default: return cudaErrorInvalidValue;                         \
+        }                                                                  \
+    }                                                                      \
+    if (mr != limb_gemm_rows_per_limb(na)) return cudaErrorInvalidValue;  \
     switch (na * 10 + nb) {                                                \
         case 11: return FN<1, 1>(__VA_ARGS__);                             \
         case 21: return FN<2, 1>(__VA_ARGS__);                             \
@@ -432,9 +356,27 @@ bool limb_gemm_supported(int na, int nb) {
 
 int limb_gemm_rows_per_limb(int na) { return na <= 2 ? 128 : 64; }
 
-cudaError_t limb_gemm_prepare(int na, int nb) { QX_LIMB_DISPATCH(prepare_t) }
+// Rows per limb for an output of m_extent M-side rows by n_extent N-side
+// rows on num_sms SMs.  Halving the tile height halves each tile's MMAs,
+// drains and stores but doubles the tiles; it pays when the rounds of
+// half-height tiles (each counted at 0.6 of a full tile, for the per-tile
+// fixed costs) take less than the rounds of full ones -- small problems and
+// problems whose last round of full tiles is mostly empty.
+int limb_gemm_pick_rows(int na, int64_t m_extent, int64_t n_extent, int num_sms) {
+    const int mr = limb_gemm_rows_per_limb(na);
+    if (na > 2 || num_sms < 1) return mr;
+    const int64_t tm = (m_extent + kBM - 1) / kBM;
+    const int64_t full = tm * ((n_extent + mr - 1) / mr);
+    const int64_t half = tm * ((n_extent + 63) / 64);
+    const int64_t r_full = (full + num_sms - 1) / num_sms;
+    const int64_t r_half = (half + num_sms - 1) / num_sms;
+    return 0.6 * double(r_half) < double(r_full) ? 64 : mr;
+}
+
+cudaError_t limb_gemm_prepare(int na, int nb, int mr) { QX_LIMB_DISPATCH(prepare_t) }
 
 cudaError_t limb_gemm_launch(int na, int nb, const MmaArgs &a, int grid, cudaStream_t stream) {
+    const int mr = a.mr;
     QX_LIMB_DISPATCH(launch_t, a, grid, stream)
 }
 

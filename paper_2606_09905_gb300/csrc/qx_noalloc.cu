@@ -35,8 +35,12 @@
 
 namespace qx {
 bool plan_contraction(qx_range rn, qx_range rm, int64_t K, Scheme *best);
+int limb_gemm_pick_rows(int na, int64_t m_extent, int64_t n_extent, int num_sms);
 int limb_gemm_rows_per_limb(int na);
-cudaError_t limb_gemm_prepare(int na, int nb);
+bool fused_gemm_packed_ok(int na, int shift_n, int nb, int shift_m, bool values_fit_int16);
+cudaError_t fused_gemm_prepare(int na, int nb, bool i32, bool pk);
+cudaError_t fused_gemm_launch(int na, int nb, bool i32, bool pk, const MmaArgs &a, int grid, cudaStream_t stream);
+cudaError_t limb_gemm_prepare(int na, int nb, int mr);
 cudaError_t limb_gemm_launch(int na, int nb, const MmaArgs &a, int grid, cudaStream_t stream);
 cudaError_t launch_pack_gemm(bool i32, const void *A, const void *B, int64_t lda, int64_t ldb,
                              int M, int N, int K, int Kp, __half *a_planes, __half *bt_planes,
@@ -166,10 +170,14 @@ extern "C" qx_status qx_gemm_i16_i32_noalloc(int64_t M, int64_t N, int64_t K, qx
     const size_t a_bytes = size_t(na) * size_t(M) * size_t(Kp) * 2;
     const size_t b_bytes = size_t(nb) * size_t(N) * size_t(Kp) * 2;
     const size_t need = 256 + round256(a_bytes) + round256(b_bytes);
-    if (need > kScratchBytes)
+    // Planes that do not fit the scratch: the fused kernel needs none (rows
+    // of A and B must start on 16-byte boundaries, K and N multiples of 8).
+    const bool fused = need > kScratchBytes;
+    if (fused && (K % 8 != 0 || N % 8 != 0))
         return refuse(QX_ERR_UNSUPPORTED,
-                      "this GEMM needs %zu bytes of scratch; the static scratch holds %zu bytes "
-                      "(use the plan-based qx_gemm_i16_i32 for larger problems)",
+                      "this GEMM needs %zu bytes of scratch; the static scratch holds %zu bytes, "
+                      "and the scratch-free fused path needs K and N multiples of 8 "
+                      "(use the plan-based qx_gemm_i16_i32)",
                       need, kScratchBytes);
 
     int dev = 0;
@@ -204,9 +212,48 @@ extern "C" qx_status qx_gemm_i16_i32_noalloc(int64_t M, int64_t N, int64_t K, qx
         return QX_OK;
     }
 
+    if (fused) {
+        MmaArgs f;
+        memset(&f, 0, sizeof f);
+        f.out = C;
+        f.err = err;
+        f.out_row_stride = N;
+        f.mode = 0;
+        f.m_extent = int(N);
+        f.n_extent = int(M);
+        f.kblocks = int((K + kBK - 1) / kBK);
+        f.chunk_kb = int(s.chunk_kb);
+        f.mr = limb_gemm_rows_per_limb(na);
+        f.tiles_m = int((N + kBM - 1) / kBM);
+        f.tiles_n = int((M + f.mr - 1) / f.mr);
+        f.group_n = f.tiles_n < 16 ? f.tiles_n : 16;
+        f.shift_n = s.n.shift;
+        f.shift_m = s.m.shift;
+        f.raw_a = A;
+        f.raw_b = B;
+        f.lda = K;
+        f.ldb = N;
+        f.K = int(K);
+        f.chk = (flags & QX_FLAG_CHECK_RANGES) ? 1 : 0;
+        f.lo_a = range_a.lo;
+        f.hi_a = range_a.hi;
+        f.lo_b = range_b.lo;
+        f.hi_b = range_b.hi;
+        const bool pk = fused_gemm_packed_ok(na, s.n.shift, nb, s.m.shift, true);
+        const int ftiles = f.tiles_m * f.tiles_n;
+        cudaError_t e = fused_gemm_prepare(na, nb, false, pk);
+        if (e == cudaSuccess)
+            e = fused_gemm_launch(na, nb, false, pk, f, ftiles < num_sms ? ftiles : num_sms, cs);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return refuse(QX_ERR_CUDA, "launch failed: %s", cudaGetErrorString(e));
+        }
+        return QX_OK;
+    }
+
     __half *a_planes = reinterpret_cast<__half *>(static_cast<char *>(base) + 256);
     __half *bt_planes = reinterpret_cast<__half *>(static_cast<char *>(base) + 256 + round256(a_bytes));
-    const int mr = limb_gemm_rows_per_limb(na);
+    const int mr = limb_gemm_pick_rows(na, N, M, num_sms);
 
     MmaArgs a;
     memset(&a, 0, sizeof a);
@@ -237,10 +284,11 @@ extern "C" qx_status qx_gemm_i16_i32_noalloc(int64_t M, int64_t N, int64_t K, qx
     a.group_n = a.tiles_n < 16 ? a.tiles_n : 16;
     a.shift_n = s.n.shift;
     a.shift_m = s.m.shift;
+    a.mr = mr;
     const int tiles = a.tiles_m * a.tiles_n;
     const int grid = tiles < num_sms ? tiles : num_sms;
 
-    cudaError_t e = limb_gemm_prepare(na, nb);
+    cudaError_t e = limb_gemm_prepare(na, nb, mr);
     if (e == cudaSuccess)
         e = launch_pack_gemm(false, A, B, K, N, int(M), int(N), int(K), int(Kp), a_planes, bt_planes,
                              na, s.n.shift, nb, s.m.shift, (flags & QX_FLAG_CHECK_RANGES) ? 1 : 0,

@@ -1,0 +1,123 @@
+// qx_tile.cuh -- tile geometry and epilogue of the tiled limb GEMM, shared by
+// the kernel that reads packed FP16 limb planes (qx_mma.cu) and the kernel
+// that converts integer operands to limbs on the fly (qx_fused.cu).
+#pragma once
+
+#include "qx_device.cuh"
+#include "qx_internal.h"
+
+namespace qx {
+
+// MR_: N-side rows per limb.  128 by default (64 with more than two limbs,
+// which keeps the MMA's N = limbs x MR within 256); 64 for one or two limbs
+// when a problem has too few 128-row tiles to fill the SMs.
+template <int NA, int NB, int KIND, int MR_ = (NA <= 2 ? 128 : 64)>
+struct TileCfg {
+    static constexpr bool TF = KIND == kKindTf32x3;
+    static constexpr int MR = MR_;                  // N-side rows per limb
+    static constexpr int UN = NA * MR;              // MMA N
+    static constexpr int M_TILE = kBM * 128;        // bytes of one M-side limb tile
+    static constexpr int N_TILE = UN * 128;         // bytes of the stacked N-side tile
+    static constexpr int STAGE = NB * M_TILE + N_TILE;
+    static constexpr int STAGES_FIT = (200 * 1024) / STAGE;
+    static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
+    // TMEM columns per accumulator set: every M-side limb has its own for the
+    // exact kind; the TF32 kind sums all products into one.
+    static constexpr int ACC_COLS = TF ? UN : NB * UN;
+    static constexpr int NBUF = ACC_COLS <= 256 ? 2 : 1;
+    static constexpr int TMEM_NEED = ACC_COLS * NBUF;
+    static constexpr int TMEM_COLS = TMEM_NEED <= 32    ? 32
+                                     : TMEM_NEED <= 64  ? 64
+                                     : TMEM_NEED <= 128 ? 128
+                                     : TMEM_NEED <= 256 ? 256
+                                                        : 512;
+    static constexpr int RPT = MR / 2;              // N-side rows per epilogue thread
+    static constexpr uint32_t AB_TYPE = TF ? 2u : 0u;
+    static constexpr uint32_t IDESC = make_idesc(kBM, UN, AB_TYPE);
+    static constexpr uint32_t IDESC_FIRST = make_idesc(kBM, MR, AB_TYPE);  // first N-side limb only
+    static constexpr int BK_ELEMS = TF ? kBK32 : kBK;                     // K per 128-byte row
+    static constexpr int BAR_BYTES = 256;
+    static constexpr int SMEM = STAGES * STAGE + BAR_BYTES + 1024;
+    // warp 0: M-side TMA producer; warp 1: TMEM + MMA issue; warps 2-9:
+    // epilogue; warp 10: N-side TMA producer.  One thread needs a few hundred
+    // cycles to issue a TMA load, so two producer threads keep a k-block's
+    // loads within its MMA time.
+    static constexpr int THREADS = 352;
+    static constexpr int N_PRODUCER_WARP = 10;
+    static_assert(UN % 16 == 0 && UN >= 16 && UN <= 256, "MMA N out of range");
+    static_assert(TMEM_NEED <= 512, "accumulators exceed tensor memory");
+    static_assert(RPT % 32 == 0, "epilogue works in 32-column TMEM loads");
+    static_assert(!TF || (NA == 2 && NB == 2), "TF32x3 stacks big/small on both sides");
+};
+
+// Tile order: groups of `group_n` N-side tiles, M-side tiles inside a group,
+// so the CTAs resident at one time share operand tiles through L2.
+__device__ __forceinline__ void tile_coords(int t, const MmaArgs &a, int &tm, int &tn) {
+    const int per_group = a.group_n * a.tiles_m;
+    const int g = t / per_group;
+    const int first = g * a.group_n;
+    const int gs = min(a.group_n, a.tiles_n - first);
+    const int r = t - g * per_group;
+    tn = first + r % gs;
+    tm = r / gs;
+}
+
+
+// Exact kind: add one chunk's accumulators (every M-side limb j, N-side limb
+// i) into the running wrapping int32 sums of this thread.  `tb` addresses the
+// thread's TMEM lane quarter, the accumulator set and its half of the N-side
+// rows; 32-row groups wholly past the N-side extent are skipped.
+template <int NA, int NB, int MR_>
+__device__ __forceinline__ void drain_exact(uint32_t tb, int rows_left, int shift_n, int shift_m,
+                                            uint32_t (&acc)[TileCfg<NA, NB, kKindExact, MR_>::RPT]) {
+    using T = TileCfg<NA, NB, kKindExact, MR_>;
+#pragma unroll
+    for (int j = 0; j < NB; ++j) {
+#pragma unroll
+        for (int i = 0; i < NA; ++i) {
+            const int sh = i * shift_n + j * shift_m;
+#pragma unroll
+            for (int p = 0; p < T::RPT / 32; ++p) {
+                if (p * 32 >= rows_left) continue;
+                uint32_t v[32];
+                tmem_ld32(tb + j * T::UN + i * T::MR + p * 32, v);
+                tmem_wait_ld(v);
+#pragma unroll
+                for (int x = 0; x < 32; ++x)
+                    acc[p * 32 + x] += uint32_t(__float2int_rn(__uint_as_float(v[x]))) << sh;
+            }
+        }
+    }
+}
+
+// Store a finished tile: this thread owns output column (M-side row)
+// tm*128 + q*32 + lane and N-side rows nrow0 .. nrow0 + RPT - 1.  Conv modes
+// write NCHW.  Integer kinds apply the optional ReLU-requantize first.
+template <int NA, int NB, int KIND, int MR_>
+__device__ __forceinline__ void store_tile(const MmaArgs &a, int tm, int tn, int q, int hh, int lane,
+                                           uint32_t (&acc)[TileCfg<NA, NB, KIND, MR_>::RPT]) {
+    using T = TileCfg<NA, NB, KIND, MR_>;
+    const int mrow = tm * kBM + q * 32 + lane;
+    const bool lane_ok = mrow < a.m_extent;
+    int64_t lane_off = mrow;
+    if (a.mode != 0) {   // conv: pixel mrow of image img, NCHW output
+        const int img = mrow / a.PQ;
+        lane_off = int64_t(img) * a.k_out * a.PQ + (mrow - img * a.PQ);
+    }
+    if constexpr (!T::TF) {
+        if (a.rq_on) {   // ReLU, requantizing shift, clamp
+#pragma unroll
+            for (int r = 0; r < T::RPT; ++r)
+                acc[r] = uint32_t(min(max(int32_t(acc[r]), 0) >> a.rq_shift, a.rq_hi));
+        }
+    }
+    const int nrow0 = tn * T::MR + hh * T::RPT;
+    // both output types are 32-bit: store the raw words
+    uint32_t *o = static_cast<uint32_t *>(a.out) + lane_off + int64_t(nrow0) * a.out_row_stride;
+#pragma unroll
+    for (int r = 0; r < T::RPT; ++r) {
+        if (lane_ok && nrow0 + r < a.n_extent) o[int64_t(r) * a.out_row_stride] = acc[r];
+    }
+}
+
+}  // namespace qx

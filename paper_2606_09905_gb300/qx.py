@@ -25,6 +25,8 @@ I16, I32, F32 = 0, 1, 2
 FLAG_CHECK_RANGES = 1
 FLAG_ATTN_REASSOC = 2         # attention: O = Q (K^T V), integer plans only
 FLAG_RELU_REQUANT = 4         # GEMM / conv: out = min(max(acc, 0) >> rq_shift, rq_hi)
+FLAG_FUSED_CONVERT = 8        # GEMM: one kernel converts the operands to limbs on the fly
+FLAG_PREPASS = 16             # GEMM: packing pre-pass, then the tensor-core kernel
 
 # Every function the header declares; the CPU tests check the exports.
 EXPORTS = ("qx_plan_create", "qx_plan_destroy", "qx_plan_query", "qx_plan_info",
@@ -32,7 +34,7 @@ EXPORTS = ("qx_plan_create", "qx_plan_destroy", "qx_plan_query", "qx_plan_info",
            "qx_pack", "qx_run_packed", "qx_plan_status", "qx_status_string",
            "qx_last_error", "qx_version", "qx_gemm_i16_i32_noalloc", "qx_minmax",
            "qx_pool2d", "qx_lenet_create", "qx_lenet_forward", "qx_lenet_status",
-           "qx_lenet_destroy")
+           "qx_lenet_destroy", "qx_plan_fused")
 
 
 class QxError(RuntimeError):
@@ -112,6 +114,7 @@ def load() -> ctypes.CDLL:
             "qx_lenet_forward": ([P, V, V, V, V, V, V, V, V], ctypes.c_int),
             "qx_lenet_status": ([P], ctypes.c_int),
             "qx_lenet_destroy": ([P], ctypes.c_int),
+            "qx_plan_fused": ([P], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -273,6 +276,11 @@ class Plan:
     def status(self) -> int:
         """Synchronise and return (and clear) the device error word as a status."""
         return int(load().qx_plan_status(self.handle))
+
+    @property
+    def fused(self) -> bool:
+        """True if GEMM calls run the fused single-kernel path."""
+        return load().qx_plan_fused(self.handle) == 1
 
     # -- GEMM ------------------------------------------------------------
     def _gemm(self, fn, A, B, C, stream, dt):

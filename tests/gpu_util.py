@@ -17,10 +17,17 @@ def wrap32(x: np.ndarray) -> np.ndarray:
     return ((x.astype(np.int64) + 2**31) % 2**32 - 2**31).astype(np.int64)
 
 
-def gemm_gpu(A, B, range_a, range_b, dtype=qx.I16, flags=0, stream=None):
+PATH_FLAGS = {None: 0, "fused": qx.FLAG_FUSED_CONVERT, "prepass": qx.FLAG_PREPASS}
+
+
+def gemm_gpu(A, B, range_a, range_b, dtype=qx.I16, flags=0, stream=None, path=None):
+    """C = A B through one plan; `path` forces the fused or the pre-pass GEMM."""
     M, K = A.shape
     N = B.shape[1]
+    flags |= PATH_FLAGS[path]
     with qx.Plan(qx.gemm_desc(M, N, K, range_a, range_b, dtype=dtype, flags=flags)) as plan:
+        if path is not None:
+            assert plan.fused == (path == "fused")
         fn = plan.gemm_i16_i32 if dtype == qx.I16 else plan.gemm_i32
         C = fn(A.cuda(), B.cuda(), stream=stream)
         torch.cuda.synchronize()

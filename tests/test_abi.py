@@ -149,3 +149,18 @@ def test_lenet_create_rejects_bad_arguments(lib):
     with pytest.raises(qx.QxError) as e:
         qx.Lenet(8, (0, 255), [(-7, 7)] * 5, (4, 5, 5, 5), -1, device=0)
     assert e.value.status == qx.ERR_INVALID_ARG
+
+
+def test_gemm_path_flags_validation(lib):
+    F, P = qx.FLAG_FUSED_CONVERT, qx.FLAG_PREPASS
+    for flags in (F, P):                                     # GEMM plans only
+        with pytest.raises(qx.QxError) as e:
+            qx.query(qx.conv_desc(1, 64, 8, 8, 4, 3, 3, 1, 1, (-5, 5), (-5, 5), flags=flags))
+        assert e.value.status == qx.ERR_INVALID_ARG
+    with pytest.raises(qx.QxError) as e:                     # one path at a time
+        qx.query(qx.gemm_desc(8, 8, 8, (-1, 1), (-1, 1), flags=F | P))
+    assert e.value.status == qx.ERR_INVALID_ARG
+    # either flag alone plans the same exact scheme
+    base = qx.query(qx.gemm_desc(256, 256, 256, (-1023, 1023), (-1023, 1023)))
+    assert qx.query(qx.gemm_desc(256, 256, 256, (-1023, 1023), (-1023, 1023), flags=F)) == base
+    assert qx.query(qx.gemm_desc(256, 256, 256, (-1023, 1023), (-1023, 1023), flags=P)) == base

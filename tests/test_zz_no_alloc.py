@@ -72,8 +72,22 @@ def test_noalloc_without_status_word_and_python_wrapper():
     assert torch.equal(C, _plan_result(A, B, (-500, 500), (-500, 500)))
 
 
-def test_noalloc_rejects_problems_beyond_its_scratch():
-    M = N = K = 4096                          # needs 96 MiB of planes
+def test_noalloc_beyond_its_scratch_runs_the_fused_kernel():
+    # 4096^3 needs 96 MiB of limb planes, three times the static scratch:
+    # the call takes the fused single-kernel path, which needs none
+    M = N = K = 4096
+    A, B = inputs.gemm_case(M, N, K, -500, 500, seed=11)
+    A, B = A.cuda(), B.cuda()
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    C = torch.full((M, N), 7, dtype=torch.int32, device="cuda")
+    assert _noalloc(A, B, C, (-500, 500), (-500, 500), status) == qx.OK
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert torch.equal(C, _plan_result(A, B, (-500, 500), (-500, 500)))
+
+
+def test_noalloc_rejects_unaligned_problems_beyond_its_scratch():
+    M = N = K = 4095                          # planes beyond the scratch, rows not 16-byte aligned
     A = torch.zeros((M, K), dtype=torch.int16, device="cuda")
     B = torch.zeros((K, N), dtype=torch.int16, device="cuda")
     C = torch.full((M, N), 7, dtype=torch.int32, device="cuda")
