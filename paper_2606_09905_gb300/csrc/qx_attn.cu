@@ -45,15 +45,19 @@ constexpr int kMaxCluster = 8;
 // ---------------------------------------------------------- integer kind
 // Warps 0-7 turn S into FP16 digits in place in TMEM and finally write the
 // partial O; warp 8 issues the TMA loads; warp 9 owns TMEM and issues the
-// MMAs.  A key block holds 128 keys: S_b = Q K_b^T is one N = 128 product
-// per 16 head dimensions, and O += S_b V_b takes its A operand (the digits)
-// straight from TMEM, so the digits never touch shared memory.  S has three
-// TMEM buffers for head sizes up to 64 (two for 128), so the digits of
-// block b+1 are made while the tensor cores run O += S_b V_b and S_{b+2}.
-constexpr int kThreads = 320;
+// O_lo += lo V MMAs, warp 11 the O_hi += hi V ones; warp 10 issues the
+// S = Q K^T MMAs.  A key block holds 128
+// keys: S_b = Q K_b^T is one N = 128 product per 16 head dimensions, and
+// O += S_b V_b takes its A operand (the digits) straight from TMEM, so the
+// digits never touch shared memory.  S has three TMEM buffers for head sizes
+// up to 64 (two for 128), so S_{b+1} and S_{b+2} can be computed and their
+// digits made while the tensor cores run O += S_b V_b.
+constexpr int kThreads = 384;
 constexpr int kConv = 256;
 constexpr int kProducerWarp = 8;
-constexpr int kIssuerWarp = 9;
+constexpr int kIssuerWarp = 9;                          // TMEM owner; issues O_lo += lo V
+constexpr int kSIssuerWarp = 10;                        // issues S = Q K^T
+constexpr int kHiIssuerWarp = 11;                       // issues O_hi += hi V
 constexpr int kBlockKeys = 128;                         // keys per S block
 constexpr int kMaxStages = 8;                           // K / V^T ring
 constexpr int kMaxSBufs = 3;
@@ -77,7 +81,7 @@ static_assert(Smem::RING / (Smem::K_BLK + 2 * 64 * 128) <= kMaxStages, "ring bar
 static_assert(Smem::total <= 227 * 1024, "shared memory");
 
 struct BarsI {
-    uint64_t *q, *kv_full, *kv_empty, *s_full, *sready, *o_done, *tail;
+    uint64_t *q, *kv_full, *kv_empty, *s_full, *sready, *o_done, *tail, *tail_s, *tail_hi;
     uint32_t *tmem_slot;
     volatile int *abort_flag;
     __device__ BarsI(uint8_t *base) {
@@ -91,24 +95,28 @@ struct BarsI {
         tail = o_done + kMaxSBufs;
         tmem_slot = reinterpret_cast<uint32_t *>(tail + 1);
         abort_flag = reinterpret_cast<volatile int *>(tail + 2);
+        tail_s = tail + 3;
+        tail_hi = tail + 4;
     }
     __device__ void init() {
         mbar_init(q, 1);
         for (int i = 0; i < kMaxStages; ++i) {
             mbar_init(&kv_full[i], 1);
-            mbar_init(&kv_empty[i], 1);
+            mbar_init(&kv_empty[i], 2);            // one commit per O issuer
         }
         for (int i = 0; i < kMaxSBufs; ++i) {
             mbar_init(&s_full[i], 1);
             mbar_init(&sready[i], kConv / 32);     // one arrival per converter warp
-            mbar_init(&o_done[i], 1);
+            mbar_init(&o_done[i], 2);              // one commit per O issuer
         }
         mbar_init(tail, 1);
+        mbar_init(tail_s, 1);
+        mbar_init(tail_hi, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
 };
-static_assert(1 + 2 * kMaxStages + 3 * kMaxSBufs + 1 + 2 <= 256 / 8, "barrier block");
+static_assert(1 + 2 * kMaxStages + 3 * kMaxSBufs + 1 + 4 <= 256 / 8, "barrier block");
 
 // ------------------------------------------------------------- FP32 kind
 constexpr int kTmemS = 0;                               // S block
@@ -390,24 +398,70 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
                 mbar_wait_drain(bar.q, 0);
             }
         }
-    } else if (warp == kIssuerWarp) {
-        // ---------------------------------------------------------- MMA issue
-        // The whole warp runs this loop; one elected lane issues each MMA and
+    } else if (warp == kIssuerWarp || warp == kHiIssuerWarp) {
+        // ------------------------------------------ MMA issue: O_lo, O_hi += S V
+        // Three warps issue the MMAs: S = Q K^T, O_lo += lo V and O_hi += hi V.
+        // One thread spends tens of cycles issuing each tcgen05.mma, and O's
+        // N = dp products are too short to hide that when one thread issues
+        // them all.  A commit tracks the MMAs of the thread that issues it,
+        // so each issuer commits its own (o_done and kv_empty count two).
+        // The whole warp runs the loop; one elected lane issues each MMA and
         // commit (warp-uniform operands make the issue cheaper).
         if (nb > 0) {
             const uint32_t idesc_o = make_idesc(128, dp, 0);
+            const uint32_t tacc = warp == kIssuerWarp ? tOlo : tOhi;
+            const uint32_t dig = warp == kIssuerWarp ? 0u : 16u;   // lo or hi columns
+            int o_st = 0;
+            for (int b = 0; ok && b < nb; ++b) {
+                const int i = b % nsb;
+                const int st = o_st;
+                if (++o_st == nst) o_st = 0;
+                if (!mbar_wait_warp(&bar.sready[i], uint32_t((b / nsb) & 1), bar.abort_flag, a.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint64_t vdesc = make_sdesc(smem_addr(skv + st * stage_bytes + dkb * Smem::K_BLK));
+                const uint32_t ts = tmem + uint32_t(i * kBlockKeys) + dig;
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const uint64_t vd = vdesc + uint64_t((h * dp * 128 + kk * 32) >> 4);
+                        const uint32_t col = uint32_t(64 * h + 32 * (kk >> 1) + 8 * (kk & 1));
+                        mma_f16_ts_elect(tacc, ts + col, vd, idesc_o, (b > 0 || h > 0 || kk > 0) ? 1u : 0u);
+                    }
+                // S_b finished before its digits were made, so these commits
+                // also cover the K rows of the stage
+                tc_commit_elect(&bar.o_done[i]);
+                tc_commit_elect(&bar.kv_empty[st]);
+            }
+            if (!ok) {
+                // MMAs already issued finish before TMEM and shared memory go
+                uint64_t *t = warp == kIssuerWarp ? bar.tail : bar.tail_hi;
+                tc_commit_elect(t);
+                mbar_wait_drain(t, 0);
+            }
+        }
+    } else if (warp == kSIssuerWarp) {
+        // ------------------------------------------------- MMA issue: S = Q K^T
+        if (nb > 0) {
             const uint64_t qdesc = make_sdesc(smem_addr(sq));
-            // S runs two key blocks ahead of O; each keeps its own ring position
-            int s_st = 0, s_round = 0, o_st = 0;
-            auto issue_s = [&](int b) -> bool {
+            int s_st = 0, s_round = 0;
+            ok = mbar_wait_warp(bar.q, 0, bar.abort_flag, a.err);
+            for (int b = 0; ok && b < nb; ++b) {
                 const int i = b % nsb;
                 // S_i was last read (as digits) by O of block b - nsb
                 if (b >= nsb &&
-                    !mbar_wait_warp(&bar.o_done[i], uint32_t(((b - nsb) / nsb) & 1), bar.abort_flag, a.err))
-                    return false;
+                    !mbar_wait_warp(&bar.o_done[i], uint32_t(((b - nsb) / nsb) & 1), bar.abort_flag, a.err)) {
+                    ok = false;
+                    break;
+                }
                 const int st = s_st;
-                if (!mbar_wait_warp(&bar.kv_full[st], uint32_t(s_round & 1), bar.abort_flag, a.err))
-                    return false;
+                if (!mbar_wait_warp(&bar.kv_full[st], uint32_t(s_round & 1), bar.abort_flag, a.err)) {
+                    ok = false;
+                    break;
+                }
                 if (++s_st == nst) {
                     s_st = 0;
                     ++s_round;
@@ -422,38 +476,10 @@ __global__ void __launch_bounds__(attn::kThreads, 1) attn_core_kernel(const __gr
                                       kdesc + uint64_t((kb * Smem::K_BLK + kk * 32) >> 4), kIdescS,
                                       (kb > 0 || kk > 0) ? 1u : 0u);
                 tc_commit_elect(&bar.s_full[i]);
-                return true;
-            };
-            ok = mbar_wait_warp(bar.q, 0, bar.abort_flag, a.err) && issue_s(0) && (nb < 2 || issue_s(1));
-            for (int b = 0; ok && b < nb; ++b) {
-                const int i = b % nsb;
-                const int st = o_st;
-                if (++o_st == nst) o_st = 0;
-                if (!mbar_wait_warp(&bar.sready[i], uint32_t((b / nsb) & 1), bar.abort_flag, a.err)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint64_t vdesc = make_sdesc(smem_addr(skv + st * stage_bytes + dkb * Smem::K_BLK));
-                const uint32_t ts = tmem + uint32_t(i * kBlockKeys);
-#pragma unroll
-                for (int h = 0; h < 2; ++h)
-#pragma unroll
-                    for (int kk = 0; kk < 4; ++kk) {
-                        const uint64_t vd = vdesc + uint64_t((h * dp * 128 + kk * 32) >> 4);
-                        const uint32_t col = uint32_t(64 * h + 32 * (kk >> 1) + 8 * (kk & 1));
-                        const uint32_t acc = (b > 0 || h > 0 || kk > 0) ? 1u : 0u;
-                        mma_f16_ts_elect(tOlo, ts + col, vd, idesc_o, acc);
-                        mma_f16_ts_elect(tOhi, ts + col + 16u, vd, idesc_o, acc);
-                    }
-                tc_commit_elect(&bar.o_done[i]);
-                tc_commit_elect(&bar.kv_empty[st]);
-                if (b + 2 < nb && !issue_s(b + 2)) ok = false;
             }
             if (!ok) {
-                // MMAs already issued finish before TMEM and shared memory go
-                tc_commit_elect(bar.tail);
-                mbar_wait_drain(bar.tail, 0);
+                tc_commit_elect(bar.tail_s);
+                mbar_wait_drain(bar.tail_s, 0);
             }
         }
     } else {
