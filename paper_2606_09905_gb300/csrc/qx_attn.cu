@@ -119,10 +119,19 @@ struct BarsI {
 static_assert(1 + 2 * kMaxStages + 3 * kMaxSBufs + 1 + 4 <= 256 / 8, "barrier block");
 
 // ------------------------------------------------------------- FP32 kind
-constexpr int kTmemS = 0;                               // S block
+// Warps 0-3 split S into TF32 big/small parts (one query row per thread) and
+// finally write the partial O; warp 4 owns TMEM and issues the TMA loads;
+// warp 5 issues S = Q K^T and warp 6 O^T += V^T S^T.  S is double-buffered
+// in TMEM and as the split operand tile in shared memory, and so is the K /
+// V^T stage, so S of block b+1 is computed and split while the tensor cores
+// run O of block b.
+constexpr int kTmemS = 0;                               // S blocks: 2 x 64 columns
 constexpr int kTmemO = 256;                             // O^T: two halves of 128 queries
-constexpr int kThreads32 = 160;     // warps 0-3: S conversion and epilogue; warp 4: TMA + MMA
+constexpr int kThreads32 = 224;
 constexpr int kConv32 = 128;
+constexpr int kLoadWarp32 = 4;
+constexpr int kSWarp32 = 5;
+constexpr int kOWarp32 = 6;
 constexpr int kKeys32 = 32;
 constexpr int kDp32 = 64;                               // head size padded to 64
 constexpr uint32_t kIdescS32 = make_idesc(128, 2 * kKeys32, 2);
@@ -134,54 +143,51 @@ struct Smem32 {
     static constexpr int K_KQ = 2 * kKeys32 * 128;      // one 32-wide k-block, big + small
     static constexpr int VT = 2 * 128 * 128;            // big + small, 128 rows, 32 keys
     static constexpr int KV_STAGE = 2 * K_KQ + VT;
-    static constexpr int S = 2 * kQTile * 128;
+    static constexpr int S = 2 * kQTile * 128;          // split S tile, big + small
     static constexpr int q_off = 0;
     static constexpr int kv_off = 2 * Q_KQ;
-    static constexpr int s_off = kv_off + 2 * KV_STAGE;
-    static constexpr int part_off = s_off;              // partial O reuses the S tile at the end
-    static constexpr int bar_off = s_off + S;
+    static constexpr int s_off = kv_off + 2 * KV_STAGE; // two S tiles
+    static constexpr int part_off = s_off;              // partial O reuses S tile 0 at the end
+    static constexpr int bar_off = s_off + 2 * S;
     static constexpr int total = bar_off + 256 + 1024;
 };
 static_assert(kQTile * kDp32 * 4 <= Smem32::S, "FP32 partial must fit the S tile");
+static_assert(Smem32::total <= 227 * 1024, "FP32 shared memory");
 
 struct Bars {
-    uint64_t *q, *kv, *s, *sready, *o, *tail;
+    uint64_t *q, *kv_full, *kv_empty, *s_full, *s_free, *sready, *o_done, *tail_s, *tail_o;
     uint32_t *tmem_slot;
     volatile int *abort_flag;
     __device__ Bars(uint8_t *base) {
         uint64_t *b = reinterpret_cast<uint64_t *>(base);
         q = b;
-        kv = b + 1;   // [2]
-        s = b + 3;
-        sready = b + 4;
-        o = b + 5;
-        tail = b + 6;
-        tmem_slot = reinterpret_cast<uint32_t *>(b + 8);
-        abort_flag = reinterpret_cast<volatile int *>(b + 9);
+        kv_full = b + 1;     // [2]
+        kv_empty = b + 3;    // [2]
+        s_full = b + 5;      // [2]
+        s_free = b + 7;      // [2]
+        sready = b + 9;      // [2]
+        o_done = b + 11;     // [2]
+        tail_s = b + 13;
+        tail_o = b + 14;
+        tmem_slot = reinterpret_cast<uint32_t *>(b + 15);
+        abort_flag = reinterpret_cast<volatile int *>(b + 16);
     }
     __device__ void init() {
         mbar_init(q, 1);
-        mbar_init(&kv[0], 1);
-        mbar_init(&kv[1], 1);
-        mbar_init(s, 1);
-        mbar_init(sready, kConv32 / 32);   // one arrival per converter warp
-        mbar_init(o, 1);
-        mbar_init(tail, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&kv_full[i], 1);
+            mbar_init(&kv_empty[i], 1);
+            mbar_init(&s_full[i], 1);
+            mbar_init(&s_free[i], kConv32 / 32);   // one arrival per converter warp
+            mbar_init(&sready[i], kConv32 / 32);
+            mbar_init(&o_done[i], 1);
+        }
+        mbar_init(tail_s, 1);
+        mbar_init(tail_o, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
 };
-
-// After an abort: let issued MMAs and copies land before resources go away.
-__device__ __forceinline__ void drain_after_abort(const Bars &b, int issued_kv) {
-    tc_commit(b.tail);
-    mbar_wait_drain(b.tail, 0);
-    for (int s = 0; s < 2; ++s) {
-        const int uses = issued_kv / 2 + (s < issued_kv % 2 ? 1 : 0);
-        if (uses > 0) mbar_wait_drain(&b.kv[s], uint32_t((uses - 1) & 1));
-    }
-    mbar_wait_drain(b.q, 0);
-}
 
 // Cluster reduction of the key splits, by pushing.  The 128 query rows are
 // owned round the cluster, rows_per = ceil(128 / cs) per CTA.  After a cluster
@@ -641,7 +647,7 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
     if (nkb < 0) nkb = 0;
 
     if (threadIdx.x == 0) bar.init();
-    if (warp == 4) {
+    if (warp == kLoadWarp32) {
         tmem_alloc(bar.tmem_slot, kTmemCols);
         tmem_relinquish();
     }
@@ -649,12 +655,12 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *bar.tmem_slot;
-    const uint32_t tS = tmem + kTmemS;
     const uint32_t tO = tmem + kTmemO;
     pdl_wait();   // packed operands come from the kernel launched just before
 
     bool ok = true;
-    if (warp == 4) {
+    if (warp == kLoadWarp32) {
+        // ---------------------------------------------------------- TMA loads
         if (lane == 0 && nkb > 0) {
             tma_prefetch(&a.tm_q);
             tma_prefetch(&a.tm_k);
@@ -662,36 +668,44 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
             mbar_expect_tx(bar.q, 2 * Smem32::Q_KQ);
             for (int kq = 0; kq < 2; ++kq)
                 tma_load_3d(sq + kq * Smem32::Q_KQ, &a.tm_q, bar.q, kq * 32, qt * kQTile, 2 * hd);
-            auto load_kv = [&](int b) {
-                uint8_t *st = skv + (b & 1) * Smem32::KV_STAGE;
-                const int key0 = key_begin + b * kKeys32;
-                mbar_expect_tx(&bar.kv[b & 1], Smem32::KV_STAGE);
-                for (int kq = 0; kq < 2; ++kq)
-                    tma_load_3d(st + kq * Smem32::K_KQ, &a.tm_k, &bar.kv[b & 1], kq * 32, key0, 2 * hd);
-                tma_load_3d(st + 2 * Smem32::K_KQ, &a.tm_vt, &bar.kv[b & 1], key0, 0, 2 * hd);
-            };
-            load_kv(0);
-            int issued_kv = 1;
-            for (int b = 0; ok && b < nkb; ++b) {
-                if (b + 1 < nkb) {
-                    if (b >= 1 && !mbar_wait(bar.o, uint32_t((b - 1) & 1), bar.abort_flag, a.err)) {
-                        ok = false;
-                        break;
-                    }
-                    load_kv(b + 1);
-                    ++issued_kv;
-                }
-                if (b == 0 && !mbar_wait(bar.q, 0, bar.abort_flag, a.err)) {
-                    ok = false;
+            int issued = 0;
+            for (int b = 0; b < nkb; ++b) {
+                const int st = b & 1;
+                // the stage was last used by block b - 2, released after its O
+                if (b >= 2 && !mbar_wait(&bar.kv_empty[st], uint32_t(((b - 2) >> 1) & 1), bar.abort_flag, a.err))
                     break;
+                uint8_t *dst = skv + st * Smem32::KV_STAGE;
+                const int key0 = key_begin + b * kKeys32;
+                mbar_expect_tx(&bar.kv_full[st], Smem32::KV_STAGE);
+                for (int kq = 0; kq < 2; ++kq)
+                    tma_load_3d(dst + kq * Smem32::K_KQ, &a.tm_k, &bar.kv_full[st], kq * 32, key0, 2 * hd);
+                tma_load_3d(dst + 2 * Smem32::K_KQ, &a.tm_vt, &bar.kv_full[st], key0, 0, 2 * hd);
+                ++issued;
+            }
+            if (*bar.abort_flag) {
+                // every copy already issued lands before shared memory goes
+                for (int st = 0; st < 2; ++st) {
+                    const int uses = issued / 2 + (st < issued % 2 ? 1 : 0);
+                    if (uses > 0) mbar_wait_drain(&bar.kv_full[st], uint32_t((uses - 1) & 1));
                 }
-                if (!mbar_wait(&bar.kv[b & 1], uint32_t((b >> 1) & 1), bar.abort_flag, a.err)) {
+                mbar_wait_drain(bar.q, 0);
+            }
+        }
+    } else if (warp == kSWarp32) {
+        // ---------------------------------------------- MMA issue: S = Q K^T
+        if (lane == 0 && nkb > 0) {
+            ok = mbar_wait(bar.q, 0, bar.abort_flag, a.err);
+            const uint32_t qa = smem_addr(sq);
+            for (int b = 0; ok && b < nkb; ++b) {
+                const int st = b & 1;
+                if (!mbar_wait(&bar.kv_full[st], uint32_t((b >> 1) & 1), bar.abort_flag, a.err) ||
+                    (b >= 2 && !mbar_wait(&bar.s_free[st], uint32_t(((b - 2) >> 1) & 1), bar.abort_flag, a.err))) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t qa = smem_addr(sq);
-                const uint32_t ka = smem_addr(skv + (b & 1) * Smem32::KV_STAGE);
+                const uint32_t ka = smem_addr(skv + st * Smem32::KV_STAGE);
+                const uint32_t tS = tmem + kTmemS + uint32_t(st * 2 * kKeys32);
                 for (int kq = 0; kq < 2; ++kq)
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk) {
@@ -700,44 +714,67 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
                         mma_tf32(tS, make_sdesc(qb), kd, kIdescS32, (kq > 0 || kk > 0) ? 1u : 0u);
                         mma_tf32(tS, make_sdesc(qb + kQTile * 128), kd, kIdescS32First, 1u);
                     }
-                tc_commit(bar.s);
-                if (!mbar_wait(bar.sready, uint32_t(b & 1), bar.abort_flag, a.err)) {
+                tc_commit(&bar.s_full[st]);
+            }
+            if (!ok) {
+                tc_commit(bar.tail_s);
+                mbar_wait_drain(bar.tail_s, 0);
+            }
+        }
+    } else if (warp == kOWarp32) {
+        // ------------------------------------------ MMA issue: O^T += V^T S^T
+        if (lane == 0 && nkb > 0) {
+            for (int b = 0; ok && b < nkb; ++b) {
+                const int st = b & 1;
+                if (!mbar_wait(&bar.sready[st], uint32_t((b >> 1) & 1), bar.abort_flag, a.err)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t va = ka + 2 * Smem32::K_KQ;
-                const uint32_t sa = smem_addr(ss);
+                const uint32_t va = smem_addr(skv + st * Smem32::KV_STAGE) + 2 * Smem32::K_KQ;
+                const uint32_t sa = smem_addr(ss + st * Smem32::S);
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
                     const uint64_t sd = make_sdesc(sa + kk * 32);
                     mma_tf32(tO, make_sdesc(va + kk * 32), sd, kIdescO32, (b > 0 || kk > 0) ? 1u : 0u);
                     mma_tf32(tO, make_sdesc(va + 128 * 128 + kk * 32), sd, kIdescO32First, 1u);
                 }
-                tc_commit(bar.o);
+                // S_b finished before it was split, so this also frees K
+                tc_commit(&bar.o_done[st]);
+                tc_commit(&bar.kv_empty[st]);
             }
-            if (!ok) drain_after_abort(bar, issued_kv);
+            if (!ok) {
+                tc_commit(bar.tail_o);
+                mbar_wait_drain(bar.tail_o, 0);
+            }
         }
     } else {
         // ---------------------------------------- S -> TF32 big/small in smem
         const int row = warp * 32 + lane;
         for (int b = 0; b < nkb; ++b) {
-            if (!mbar_wait(bar.s, uint32_t(b & 1), bar.abort_flag, a.err)) {
-                ok = false;
-                break;
-            }
-            if (b >= 1 && !mbar_wait(bar.o, uint32_t((b - 1) & 1), bar.abort_flag, a.err)) {
+            const int st = b & 1;
+            if (!mbar_wait(&bar.s_full[st], uint32_t((b >> 1) & 1), bar.abort_flag, a.err)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
+            const uint32_t tS = tmem + kTmemS + uint32_t(st * 2 * kKeys32) + (uint32_t(warp * 32) << 16);
             uint32_t v0[32], v1[32];
-            tmem_ld32(tS + (uint32_t(warp * 32) << 16), v0);
-            tmem_ld32(tS + (uint32_t(warp * 32) << 16) + kKeys32, v1);
+            tmem_ld32(tS, v0);
+            tmem_ld32(tS + kKeys32, v1);
             tmem_wait_ld(v0);
             tmem_wait_ld(v1);
-            uint8_t *rbig = ss + row * 128;
-            uint8_t *rsmall = ss + (kQTile + row) * 128;
+            // the TMEM S buffer may take block b + 2 now
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bar.s_free[st]);
+            // the shared S tile was last read by O of block b - 2
+            if (b >= 2 && !mbar_wait(&bar.o_done[st], uint32_t(((b - 2) >> 1) & 1), bar.abort_flag, a.err)) {
+                ok = false;
+                break;
+            }
+            uint8_t *rbig = ss + st * Smem32::S + row * 128;
+            uint8_t *rsmall = rbig + kQTile * 128;
 #pragma unroll
             for (int c = 0; c < 8; ++c) {
                 __align__(16) float big[4], small[4];
@@ -750,14 +787,14 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
                 *reinterpret_cast<uint4 *>(rsmall + pos) = *reinterpret_cast<uint4 *>(small);
             }
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar.sready);
+            if (lane == 0) mbar_arrive(&bar.sready[st]);
         }
         // ------------------------------- this CTA's partial O -> shared memory
         // (the S tile is free once the last O MMA has completed)
         const int c = warp * 32 + lane;
-        const bool have = ok && nkb > 0 && mbar_wait(bar.o, uint32_t((nkb - 1) & 1), bar.abort_flag, a.err);
+        const bool have = ok && nkb > 0 &&
+                          mbar_wait(&bar.o_done[(nkb - 1) & 1], uint32_t(((nkb - 1) >> 1) & 1), bar.abort_flag, a.err);
         if (have) tc_fence_after();
         if (warp * 32 < kDp32) {
 #pragma unroll 1
@@ -795,7 +832,7 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
         cluster_pull_reduce_store<true>(part, kDp32, cs, qt, hd, a);
         cluster_sync();
     }
-    if (warp == 4) {
+    if (warp == kLoadWarp32) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
     }
