@@ -19,7 +19,8 @@
 // output column, which makes every warp store 32 consecutive int32 values.
 //
 // Roles (one CTA per SM, persistent over output tiles):
-//   warp 0      TMA producer (one thread): stage ring of `STAGES` buffers
+//   warps 0, 11 M-side TMA producers (one thread each, alternate k-blocks)
+//   warp 10     N-side TMA producer: stage ring of `STAGES` buffers
 //   warp 1      TMEM owner and MMA issuer (one thread)
 //   warps 2..9  epilogue: two warps per TMEM lane quarter, each owning half
 //               of the N-side rows; running int32 sums live in registers.
@@ -42,7 +43,7 @@
 namespace qx {
 
 template <int NA, int NB, int KIND, int MR_>
-__global__ void __launch_bounds__(352, 1) limb_gemm_kernel(const __grid_constant__ MmaArgs a) {
+__global__ void __launch_bounds__(384, 1) limb_gemm_kernel(const __grid_constant__ MmaArgs a) {
     using T = TileCfg<NA, NB, KIND, MR_>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -88,12 +89,15 @@ __global__ void __launch_bounds__(352, 1) limb_gemm_kernel(const __grid_constant
     // the packed operands come from the kernel launched just before this one
     pdl_wait();
 
-    if (warp == 0) {
+    if (warp == 0 || warp == T::M_PRODUCER2_WARP) {
         if (lane == 0) {
-            // ------------------------------------------------ TMA producer
-            int stage = 0;
-            uint32_t phase = 0;
-            long long issued = 0;
+            // ---------------------------------------- TMA producers, M side
+            // Two threads share the M-side loads, alternate k-blocks each: one
+            // thread spends hundreds of cycles issuing a TMA load (an im2col
+            // box more than a tiled one), which would hold a conv's k-loop.
+            // k-block g of the CTA's whole sequence goes to stage g % STAGES.
+            const int par = warp == 0 ? 0 : 1;
+            long long g = 0, last = -1;
             bool ok = true;
             for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
                 int tm, tn;
@@ -106,7 +110,10 @@ __global__ void __launch_bounds__(352, 1) limb_gemm_kernel(const __grid_constant
                     oh = rem / a.Q;
                     ow = rem - oh * a.Q;
                 }
-                for (int kb = 0; kb < a.kblocks; ++kb) {
+                for (int kb = 0; kb < a.kblocks; ++kb, ++g) {
+                    if ((g & 1) != par) continue;
+                    const int stage = int(g % T::STAGES);
+                    const uint32_t phase = uint32_t((g / T::STAGES) & 1);
                     if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, a.err)) {
                         ok = false;
                         break;
@@ -130,31 +137,23 @@ __global__ void __launch_bounds__(352, 1) limb_gemm_kernel(const __grid_constant
                                                oh * a.stride - a.pad, img, uint16_t(s),
                                                uint16_t(r));
                     }
-                    ++issued;
-                    if (++stage == T::STAGES) {
-                        stage = 0;
-                        phase ^= 1;
-                    }
+                    last = g;
                 }
             }
-            if (ok) {
+            if (ok && par == 0) {
                 // Every stage must be released by the MMA before the CTA exits,
                 // so that no commit lands on the barriers of a later CTA.
-                for (int i = 0; i < T::STAGES; ++i) {
-                    if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, a.err)) break;
-                    if (++stage == T::STAGES) {
-                        stage = 0;
-                        phase ^= 1;
-                    }
+                for (long long e = g; e < g + T::STAGES; ++e) {
+                    if (!mbar_wait(&empty[e % T::STAGES], uint32_t(((e / T::STAGES) & 1) ^ 1), abort_flag,
+                                   a.err))
+                        break;
                 }
             }
             if (*abort_flag) {
-                // Let every copy already issued land before shared memory goes.
-                for (int s = 0; s < T::STAGES; ++s) {
-                    const long long uses =
-                        issued / T::STAGES + (s < issued % T::STAGES ? 1 : 0);
-                    if (uses > 0) mbar_wait_drain(&full[s], uint32_t((uses - 1) & 1));
-                }
+                // Let every copy this thread issued land before shared memory
+                // goes: the last use of each stage it filled.
+                for (long long e = last; e >= 0 && e > last - 2 * T::STAGES; e -= 2)
+                    mbar_wait_drain(&full[e % T::STAGES], uint32_t((e / T::STAGES) & 1));
             }
         }
     } else if (warp == 1) {

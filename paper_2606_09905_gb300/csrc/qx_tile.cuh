@@ -38,12 +38,13 @@ struct TileCfg {
     static constexpr int BK_ELEMS = TF ? kBK32 : kBK;                     // K per 128-byte row
     static constexpr int BAR_BYTES = 256;
     static constexpr int SMEM = STAGES * STAGE + BAR_BYTES + 1024;
-    // warp 0: M-side TMA producer; warp 1: TMEM + MMA issue; warps 2-9:
-    // epilogue; warp 10: N-side TMA producer.  One thread needs a few hundred
-    // cycles to issue a TMA load, so two producer threads keep a k-block's
-    // loads within its MMA time.
-    static constexpr int THREADS = 352;
+    // warps 0 and 11: M-side TMA producers (alternate k-blocks); warp 1: TMEM
+    // + MMA issue; warps 2-9: epilogue; warp 10: N-side TMA producer.  One
+    // thread needs a few hundred cycles to issue a TMA load, so three
+    // producer threads keep a k-block's loads within its MMA time.
+    static constexpr int THREADS = 384;
     static constexpr int N_PRODUCER_WARP = 10;
+    static constexpr int M_PRODUCER2_WARP = 11;
     static_assert(UN % 16 == 0 && UN >= 16 && UN <= 256, "MMA N out of range");
     static_assert(TMEM_NEED <= 512, "accumulators exceed tensor memory");
     static_assert(RPT % 32 == 0, "epilogue works in 32-column TMEM loads");
