@@ -17,11 +17,22 @@
 
 namespace qx {
 
+// Range checks run after all of a thread's loads have been issued: a test
+// can end in an atomic, and a load placed after one waits for the branch
+// before it, so interleaving them would serialise the loads' round trips.
 struct RangeCheck {
     int on;
     int64_t lo, hi;
     __device__ __forceinline__ void test(int32_t v, int *err) const {
         if (on && (v < lo || v > hi)) atomicCAS(err, 0, kErrContract);
+    }
+    // the first `valid` of v
+    __device__ __forceinline__ void test8(const int32_t (&v)[8], int valid, int *err) const {
+        if (!on) return;
+        bool bad = false;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) bad |= e < valid && (v[e] < lo || v[e] > hi);
+        if (bad) atomicCAS(err, 0, kErrContract);
     }
 };
 
@@ -99,9 +110,7 @@ __global__ void __launch_bounds__(256) pack_gemm_kernel(const GemmPackArgs p) {
             const int valid = min(8, p.K - k);
             int32_t v[8];
             load8<T>(A + int64_t(row) * p.lda + k, p.vec_a && valid == 8, valid, v);
-#pragma unroll
-            for (int e = 0; e < 8; ++e)
-                if (e < valid) p.ca.test(v[e], p.err);
+            p.ca.test8(v, valid, p.err);
             store_limbs8<NA>(p.a_planes + int64_t(row) * p.Kp + k, plane_stride, v, p.shift_a);
         }
         return;
@@ -118,9 +127,7 @@ __global__ void __launch_bounds__(256) pack_gemm_kernel(const GemmPackArgs p) {
         if (k < p.K && n < p.N) {
             const int valid = min(8, p.N - n);
             load8<T>(B + int64_t(k) * p.ldb + n, p.vec_b && valid == 8, valid, v);
-#pragma unroll
-            for (int e = 0; e < 8; ++e)
-                if (e < valid) p.cb.test(v[e], p.err);
+            p.cb.test8(v, valid, p.err);
         } else {
 #pragma unroll
             for (int e = 0; e < 8; ++e) v[e] = 0;
@@ -179,9 +186,7 @@ __global__ void __launch_bounds__(256) pack_conv_kernel(const ConvPackArgs p) {
             if (c0 + cr < p.c && hw < HW) {
                 const int valid = min(8, HW - hw);
                 load8<T>(X + (int64_t(img) * p.c + c0 + cr) * HW + hw, p.vec_x && valid == 8, valid, v);
-#pragma unroll
-                for (int e = 0; e < 8; ++e)
-                    if (e < valid) p.cx.test(v[e], p.err);
+                p.cx.test8(v, valid, p.err);
             } else {
 #pragma unroll
                 for (int e = 0; e < 8; ++e) v[e] = 0;
@@ -216,12 +221,9 @@ __global__ void __launch_bounds__(256) pack_conv_kernel(const ConvPackArgs p) {
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             const int c = cg * 8 + e;
-            v[e] = 0;
-            if (c < p.c) {
-                v[e] = int32_t(W[(int64_t(o) * p.c + c) * RS + tap]);
-                p.cw.test(v[e], p.err);
-            }
+            v[e] = c < p.c ? int32_t(W[(int64_t(o) * p.c + c) * RS + tap]) : 0;
         }
+        p.cw.test8(v, p.c - cg * 8, p.err);
         store_limbs8<NW>(p.w_planes + (int64_t(o) * RS + tap) * p.Cp + cg * 8, plane_stride, v,
                          p.shift_w);
     }
@@ -289,17 +291,20 @@ __global__ void __launch_bounds__(256) pack_patches_kernel(const PatchPackArgs p
             const int w0 = ow * p.stride - p.pad;
             const T *xc = X + int64_t(img) * p.c * HW + h0 * p.wd + w0;
             int32_t v[8];
+            bool in[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
                 const int k = 8 * g + e;
                 const int tp = ktap[k];
                 const int ih = h0 + (tp >> 16);
                 const int iw = w0 + (tp & 0xffff);
-                v[e] = 0;
-                if (tp >= 0 && unsigned(ih) < unsigned(p.h) && unsigned(iw) < unsigned(p.wd)) {
-                    v[e] = int32_t(xc[koff[k]]);
-                    p.cx.test(v[e], p.err);
-                }
+                in[e] = tp >= 0 && unsigned(ih) < unsigned(p.h) && unsigned(iw) < unsigned(p.wd);
+                v[e] = in[e] ? int32_t(xc[koff[k]]) : 0;
+            }
+            if (p.cx.on) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    if (in[e]) p.cx.test(v[e], p.err);
             }
             store_limbs8<NX>(p.x_planes + int64_t(m) * p.Kp + 8 * g, plane_stride, v, p.shift_x);
         }
@@ -316,14 +321,11 @@ __global__ void __launch_bounds__(256) pack_patches_kernel(const PatchPackArgs p
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             const int k = 8 * g + e;
-            v[e] = 0;
-            if (k < RSC) {
-                const int tap = k / p.c;
-                const int ch = k - tap * p.c;
-                v[e] = int32_t(W[(int64_t(o) * p.c + ch) * RS + tap]);
-                p.cw.test(v[e], p.err);
-            }
+            const int tap = k / p.c;
+            const int ch = k - tap * p.c;
+            v[e] = k < RSC ? int32_t(W[(int64_t(o) * p.c + ch) * RS + tap]) : 0;
         }
+        p.cw.test8(v, RSC - 8 * g, p.err);
         store_limbs8<NW>(p.w_planes + int64_t(o) * p.Kp + 8 * g, plane_stride, v, p.shift_w);
     }
 }
@@ -415,6 +417,7 @@ struct AttnPackArgs {
     int *err;
     int qk_blocks;          // blocks [0, qk_blocks) pack the row operands; the rest transpose
     int v_tiles_l, v_tiles_c;
+    int vec;                // Q and K rows 16-byte aligned: 8-element vector loads
 };
 
 template <typename T>
@@ -436,15 +439,10 @@ __global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
             const int c = int(rem - row * gpr) * 8;
             const T *src = (which ? K : Q) + int64_t(row) * p.d;
             const RangeCheck &ch = which ? p.ck : p.cq;
+            const int valid = max(0, min(8, p.d - c));
             int32_t v[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                v[e] = 0;
-                if (c + e < p.d) {
-                    v[e] = int32_t(src[c + e]);
-                    ch.test(v[e], p.err);
-                }
-            }
+            load8<T>(src + c, p.vec && valid == 8, valid, v);
+            ch.test8(v, valid, p.err);
             store_limbs8<1>((which ? p.k : p.q) + int64_t(row) * p.dp + c, 0, v, 0);
         }
         return;
@@ -460,14 +458,25 @@ __global__ void __launch_bounds__(256) pack_attn_kernel(const AttnPackArgs p) {
     const T *Vh = (is_k ? K : V) + int64_t(hd) * p.L * p.d;
     __half *vth = (is_k ? p.kt : p.vt) + int64_t(hd) * p.dp * p.Lp;
     const RangeCheck &chk = is_k ? p.ck : p.cv;
-    for (int i = threadIdx.x; i < 64 * 64; i += blockDim.x) {
+    // all 16 of this thread's loads first (blockDim.x = 256)
+    int32_t v[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        const int i = threadIdx.x + 256 * j;
         const int lr = i >> 6, cc = i & 63;
-        int32_t v = 0;
-        if (l0 + lr < p.L && c0 + cc < p.d) {
-            v = int32_t(Vh[int64_t(l0 + lr) * p.d + c0 + cc]);
-            chk.test(v, p.err);
+        v[j] = (l0 + lr < p.L && c0 + cc < p.d) ? int32_t(Vh[int64_t(l0 + lr) * p.d + c0 + cc]) : 0;
+    }
+    if (chk.on) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int i = threadIdx.x + 256 * j;
+            if (l0 + (i >> 6) < p.L && c0 + (i & 63) < p.d) chk.test(v[j], p.err);
         }
-        tile[lr][cc] = v;
+    }
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        const int i = threadIdx.x + 256 * j;
+        tile[i >> 6][i & 63] = v[j];
     }
     __syncthreads();
     for (int i = threadIdx.x; i < 64 * 8; i += blockDim.x) {
@@ -728,6 +737,7 @@ cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void 
     p.ck = make_check(check, rk);
     p.cv = make_check(check, rv);
     p.err = err;
+    p.vec = (int64_t(d) * (i32 ? 4 : 2)) % 16 == 0 ? 1 : 0;   // bases are 16-byte aligned
     const int64_t qk_items = int64_t(kt ? 1 : 2) * heads * L * (dp / 8);
     int64_t qk_blocks = (qk_items + 255) / 256;
     if (qk_blocks > int64_t(num_sms) * 4) qk_blocks = int64_t(num_sms) * 4;
