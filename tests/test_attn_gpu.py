@@ -249,3 +249,14 @@ def test_attn_f32_integer_values_exact_and_deterministic():
     r1, _ = attn_gpu_f32(Qf, Kf, Vf)
     r2, _ = attn_gpu_f32(Qf, Kf, Vf)
     assert np.array_equal(r1, r2)          # fixed-order reduction of the key splits
+
+
+def test_attn_heads_f32_sampled_large():
+    # the benchmarked FP32 multi-head size, 32 heads x L = 2048: the full output
+    # on the GPU, the float64 oracle and the tolerance on three heads
+    H, L, d = 32, 2048, 64
+    Q, K, V = inputs.attn_case_f32(L, d, seed=35, heads=H)
+    got, st = attn_gpu_heads(Q, K, V, (0, 0), (0, 0), (0, 0), dtype=qx.F32)
+    assert st == qx.OK
+    for h in (0, 13, 31):
+        within_tolerance(got[h], Q[h], K[h], V[h], f"attn fp32 head {h} of 32 x 2048")

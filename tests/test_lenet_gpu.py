@@ -67,3 +67,14 @@ def test_lenet_rejects_a_range_that_could_overflow():
     with pytest.raises(qx.QxError) as e:
         qx.Lenet(4, (0, 255), [(-7, 7), (-2**20, 2**20), (-7, 7), (-7, 7), (-7, 7)], SHIFTS, ACT_HI)
     assert e.value.status == qx.ERR_CONTRACT
+
+
+def test_lenet_batch_4096_sampled():
+    # the benchmarked batch: every logit on the GPU, the oracle on a spread of
+    # images (each image's logits depend on that image alone)
+    x, *ws = inputs.lenet_case(4096, seed=4096)
+    got, st = lenet_gpu(x, ws)
+    assert st == qx.OK
+    idx = np.array([0, 1, 511, 1024, 2047, 2048, 3000, 4094, 4095])
+    want = oracle.lenet(x[torch.from_numpy(idx)], *ws, SHIFTS, ACT_HI)
+    assert_exact(got[idx], want, "lenet batch 4096, sampled images")

@@ -84,3 +84,14 @@ def test_pool_argument_errors():
         x = torch.zeros((1, 2, 4, 4), dtype=torch.int32, device="cuda")
         assert lib.qx_minmax(plan.handle, x.data_ptr(), x.data_ptr(), None) == qx.ERR_INVALID_ARG
         assert lib.qx_pool2d(plan.handle, None, x.data_ptr(), None) == qx.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("dtype,n", [(qx.I32, 1 << 28), (qx.I16, 1 << 29)])
+def test_minmax_benchmark_sizes(dtype, n):
+    # the benchmarked 1 GiB inputs, in the benchmark's launch configuration
+    x = _data((n,), dtype, seed=5)
+    with qx.Plan(qx.minmax_desc(n, dtype)) as plan:
+        out = plan.minmax(x.cuda())
+        torch.cuda.synchronize()
+        assert plan.status() == qx.OK
+    assert out.cpu().tolist() == list(oracle.minmax(x))
