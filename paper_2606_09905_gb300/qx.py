@@ -202,16 +202,28 @@ def gemm_i16_i32_noalloc(A, B, C, range_a, range_b, flags=0, dev_status=None, st
 _TORCH_DT = {I16: torch.int16, I32: torch.int32, F32: torch.float32}
 
 
-def _ptr(t: torch.Tensor, dtype: torch.dtype, shape, name: str) -> int:
+def _ptr_error(t, dtype, shape, name: str):
     if not isinstance(t, torch.Tensor) or not t.is_cuda:
         raise ValueError(f"{name} must be a CUDA tensor")
     if t.dtype != dtype:
         raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
     if shape is not None and tuple(t.shape) != tuple(shape):
         raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
-    if not t.is_contiguous():
-        raise ValueError(f"{name} must be contiguous")
-    return t.data_ptr()
+    raise ValueError(f"{name} must be contiguous")
+
+
+def _ptr(t: torch.Tensor, dtype: torch.dtype, shape, name: str) -> int:
+    """Device pointer of t after checking it is a contiguous CUDA tensor of
+    `dtype` and `shape` (a torch.Size, or None for any shape).  One combined
+    test on the common path: the binding's checks are most of a small call's
+    host time."""
+    try:
+        if (t.dtype is dtype and t.is_cuda and (shape is None or t.shape == shape)
+                and t.is_contiguous()):
+            return t.data_ptr()
+    except AttributeError:
+        pass
+    _ptr_error(t, dtype, shape, name)
 
 
 def _stream(stream) -> int:
@@ -233,6 +245,18 @@ class Plan:
         _check(lib.qx_plan_create(ctypes.byref(desc), self.device, ctypes.byref(h)),
                "qx_plan_create")
         self._h = h
+        self._lib = lib
+        # expected operand shapes, fixed by the plan
+        d = desc
+        S = torch.Size
+        if d.op == OP_GEMM:
+            self._sa = S((d.M, d.lda or d.K))
+            self._sb = S((d.K, d.ldb or d.N))
+            self._sc = S((d.M, d.ldc or d.N))
+        elif d.op == OP_CONV2D:
+            P = (d.h + 2 * d.pad - d.r) // d.stride + 1
+            Q = (d.w + 2 * d.pad - d.s) // d.stride + 1
+            self._sx, self._sw, self._sy = S((d.n, d.c, d.h, d.w)), S((d.k_out, d.c, d.r, d.s)), S((d.n, d.k_out, P, Q))
 
     @property
     def handle(self) -> ctypes.c_void_p:
@@ -284,37 +308,35 @@ class Plan:
 
     # -- GEMM ------------------------------------------------------------
     def _gemm(self, fn, A, B, C, stream, dt):
-        d = self.desc
-        lda = d.lda or d.K
-        ldb = d.ldb or d.N
-        ldc = d.ldc or d.N
         if C is None:
-            C = torch.empty((d.M, ldc), dtype=torch.int32, device=A.device)
-        a = _ptr(A, dt, (d.M, lda), "A")
-        b = _ptr(B, dt, (d.K, ldb), "B")
-        c = _ptr(C, torch.int32, (d.M, ldc), "C")
-        _check(fn(self.handle, a, b, c, _stream(stream)), fn.__name__)
+            C = torch.empty(self._sc, dtype=torch.int32, device=A.device)
+        a = _ptr(A, dt, self._sa, "A")
+        b = _ptr(B, dt, self._sb, "B")
+        c = _ptr(C, torch.int32, self._sc, "C")
+        st = fn(self.handle, a, b, c, _stream(stream))
+        if st != OK:
+            _check(st, fn.__name__)
         return C
 
     def gemm_i16_i32(self, A, B, C=None, stream=None):
-        return self._gemm(load().qx_gemm_i16_i32, A, B, C, stream, torch.int16)
+        return self._gemm(self._lib.qx_gemm_i16_i32, A, B, C, stream, torch.int16)
 
     def gemm_i32(self, A, B, C=None, stream=None):
-        return self._gemm(load().qx_gemm_i32, A, B, C, stream, torch.int32)
+        return self._gemm(self._lib.qx_gemm_i32, A, B, C, stream, torch.int32)
 
     # -- conv -------------------------------------------------------------
     def conv2d(self, x, w, y=None, stream=None):
         d = self.desc
-        P = (d.h + 2 * d.pad - d.r) // d.stride + 1
-        Q = (d.w + 2 * d.pad - d.s) // d.stride + 1
         dt = _TORCH_DT[d.in_dtype]
         out_dt = torch.float32 if d.in_dtype == F32 else torch.int32
         if y is None:
-            y = torch.empty((d.n, d.k_out, P, Q), dtype=out_dt, device=x.device)
-        px = _ptr(x, dt, (d.n, d.c, d.h, d.w), "x")
-        pw = _ptr(w, dt, (d.k_out, d.c, d.r, d.s), "w")
-        py = _ptr(y, out_dt, (d.n, d.k_out, P, Q), "y")
-        _check(load().qx_conv2d_gemm(self.handle, px, pw, py, _stream(stream)), "qx_conv2d_gemm")
+            y = torch.empty(self._sy, dtype=out_dt, device=x.device)
+        px = _ptr(x, dt, self._sx, "x")
+        pw = _ptr(w, dt, self._sw, "w")
+        py = _ptr(y, out_dt, self._sy, "y")
+        st = self._lib.qx_conv2d_gemm(self.handle, px, pw, py, _stream(stream))
+        if st != OK:
+            _check(st, "qx_conv2d_gemm")
         return y
 
     # -- min/max and pooling ------------------------------------------------
@@ -354,9 +376,12 @@ class Plan:
         shape = (d.L, d.d) if heads == 1 and Q.dim() == 2 else (heads, d.L, d.d)
         if O is None:
             O = torch.empty(shape, dtype=out_dt, device=Q.device)
-        pq, pk, pv = (_ptr(t, dt, shape, n) for t, n in ((Q, "Q"), (K, "K"), (V, "V")))
+        shape = torch.Size(shape)
+        pq, pk, pv = _ptr(Q, dt, shape, "Q"), _ptr(K, dt, shape, "K"), _ptr(V, dt, shape, "V")
         po = _ptr(O, out_dt, shape, "O")
-        _check(load().qx_attn_core(self.handle, pq, pk, pv, po, _stream(stream)), "qx_attn_core")
+        st = self._lib.qx_attn_core(self.handle, pq, pk, pv, po, _stream(stream))
+        if st != OK:
+            _check(st, "qx_attn_core")
         return O
 
 
