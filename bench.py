@@ -611,6 +611,18 @@ def run_qx(args):
                                 "gbs": round(pack_bytes / (pack_ms * 1e-3) / 1e9, 1),
                                 "hbm_peak_gbs": peaks["hbm_gbs"]}}
 
+    # Secondary roofline, the north-star's literal form: an INT8-limb design
+    # needs 4 s8 products per INT16 product, on the only INT8 tensor
+    # instruction sm_103a has (warp-level mma.sync); measured here, outside
+    # the timed regions.
+    try:
+        s8 = qx.measure_int8_mma_peak(local)
+        roofline["int8_limb"] = {"mma_sync_s8_tops": round(s8, 1), "int16_roofline_tops": round(s8 / 4, 1),
+                                 "frac_step": round(value / world / (s8 / 4), 3),
+                                 "note": "no tcgen05 INT8 kind on sm_103a; 4 s8 limb products per INT16 product"}
+    except qx.QxError as exc:
+        roofline["int8_limb"] = {"unavailable": str(exc)}
+
     extras = {}
     if not args.no_operators:
         extras = operators(torch, qx, inputs, dev)

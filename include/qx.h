@@ -312,6 +312,15 @@ qx_status qx_gemm_i16_i32_noalloc(int64_t M, int64_t N, int64_t K, qx_range rang
                                   const int16_t *B, int32_t *C, int *dev_status,
                                   qx_stream stream);
 
+/* Measurement utility (no operator uses it): the throughput, in TOPS, of the
+ * warp-level mma.sync.m16n8k32 s8 x s8 -> s32 instruction on `device`, with
+ * every SM running independent chains from registers (about a second).  An
+ * INT16 GEMM built from INT8 limbs needs four such products per INT16
+ * product, so a quarter of this is the INT8-limb roofline reported beside the
+ * FP16-digit substrate's.  sm_103a has no tcgen05 INT8 kind.  Synchronises
+ * `device`; errors: INVALID_ARG (null tops), DEVICE, CUDA. */
+qx_status qx_measure_int8_mma_peak(int device, double *tops);
+
 const char *qx_status_string(qx_status status);
 const char *qx_last_error(void);
 int qx_version(void);

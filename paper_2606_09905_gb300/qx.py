@@ -34,7 +34,7 @@ EXPORTS = ("qx_plan_create", "qx_plan_destroy", "qx_plan_query", "qx_plan_info",
            "qx_pack", "qx_run_packed", "qx_plan_status", "qx_status_string",
            "qx_last_error", "qx_version", "qx_gemm_i16_i32_noalloc", "qx_minmax",
            "qx_pool2d", "qx_lenet_create", "qx_lenet_forward", "qx_lenet_status",
-           "qx_lenet_destroy", "qx_plan_fused")
+           "qx_lenet_destroy", "qx_plan_fused", "qx_measure_int8_mma_peak")
 
 
 class QxError(RuntimeError):
@@ -115,6 +115,7 @@ def load() -> ctypes.CDLL:
             "qx_lenet_status": ([P], ctypes.c_int),
             "qx_lenet_destroy": ([P], ctypes.c_int),
             "qx_plan_fused": ([P], ctypes.c_int),
+            "qx_measure_int8_mma_peak": ([ctypes.c_int, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -224,6 +225,13 @@ def _ptr(t: torch.Tensor, dtype: torch.dtype, shape, name: str) -> int:
     except AttributeError:
         pass
     _ptr_error(t, dtype, shape, name)
+
+
+def measure_int8_mma_peak(device: int = 0) -> float:
+    """TOPS of the warp-level mma.sync s8 instruction on `device` (see qx.h)."""
+    out = ctypes.c_double(0.0)
+    _check(load().qx_measure_int8_mma_peak(int(device), ctypes.byref(out)), "qx_measure_int8_mma_peak")
+    return out.value
 
 
 def _stream(stream) -> int:

@@ -221,3 +221,11 @@ def test_gemm_requant_epilogue():
     want = oracle.requant(oracle.gemm(A, B)[0], 8, 5000)
     assert (want == 5000).any() and (want == 0).any()
     assert_exact(C.cpu().numpy().astype(np.int64), want, "gemm requant")
+
+
+def test_int8_mma_peak_measurement():
+    # the measurement utility behind the INT8-limb roofline: a positive rate,
+    # and argument errors returned without work
+    tops = qx.measure_int8_mma_peak(0)
+    assert 1.0 < tops < 1e5
+    assert qx.load().qx_measure_int8_mma_peak(0, None) == qx.ERR_INVALID_ARG
