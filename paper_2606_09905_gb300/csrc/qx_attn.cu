@@ -120,18 +120,21 @@ static_assert(1 + 2 * kMaxStages + 3 * kMaxSBufs + 1 + 4 <= 256 / 8, "barrier bl
 
 // ------------------------------------------------------------- FP32 kind
 // Warps 0-3 split S into TF32 big/small parts (one query row per thread) and
-// finally write the partial O; warp 4 owns TMEM and issues the TMA loads;
-// warp 5 issues S = Q K^T and warp 6 O^T += V^T S^T.  S is double-buffered
+// finally write the partial O; warp 4 owns TMEM and issues the Q and K loads,
+// warp 7 the V^T loads; warp 5 issues S = Q K^T and warp 6 O^T += V^T S^T.  S is double-buffered
 // in TMEM and as the split operand tile in shared memory, and so is the K /
 // V^T stage, so S of block b+1 is computed and split while the tensor cores
-// run O of block b.
+// run O of block b.  K and V^T have rings of their own (two stages each):
+// K is released by the S product, V^T by the O product, so the loads of S's
+// operands never wait for O.
 constexpr int kTmemS = 0;                               // S blocks: 2 x 64 columns
 constexpr int kTmemO = 256;                             // O^T: two halves of 128 queries
-constexpr int kThreads32 = 224;
+constexpr int kThreads32 = 256;
 constexpr int kConv32 = 128;
-constexpr int kLoadWarp32 = 4;
+constexpr int kLoadWarp32 = 4;                          // TMEM owner; Q and K loads
 constexpr int kSWarp32 = 5;
 constexpr int kOWarp32 = 6;
+constexpr int kVLoadWarp32 = 7;                         // V^T loads
 constexpr int kKeys32 = 32;
 constexpr int kDp32 = 64;                               // head size padded to 64
 constexpr uint32_t kIdescS32 = make_idesc(128, 2 * kKeys32, 2);
@@ -142,11 +145,12 @@ struct Smem32 {
     static constexpr int Q_KQ = 2 * kQTile * 128;       // one 32-wide k-block, big + small
     static constexpr int K_KQ = 2 * kKeys32 * 128;      // one 32-wide k-block, big + small
     static constexpr int VT = 2 * 128 * 128;            // big + small, 128 rows, 32 keys
-    static constexpr int KV_STAGE = 2 * K_KQ + VT;
+    static constexpr int K_STAGE = 2 * K_KQ;            // K ring stage: both 32-wide k-blocks
     static constexpr int S = 2 * kQTile * 128;          // split S tile, big + small
     static constexpr int q_off = 0;
-    static constexpr int kv_off = 2 * Q_KQ;
-    static constexpr int s_off = kv_off + 2 * KV_STAGE; // two S tiles
+    static constexpr int k_off = 2 * Q_KQ;              // K ring: 2 stages, released by S
+    static constexpr int v_off = k_off + 2 * K_STAGE;   // V^T ring: 2 stages, released by O
+    static constexpr int s_off = v_off + 2 * VT;        // two S tiles
     static constexpr int part_off = s_off;              // partial O reuses S tile 0 at the end
     static constexpr int bar_off = s_off + 2 * S;
     static constexpr int total = bar_off + 256 + 1024;
@@ -155,28 +159,32 @@ static_assert(kQTile * kDp32 * 4 <= Smem32::S, "FP32 partial must fit the S tile
 static_assert(Smem32::total <= 227 * 1024, "FP32 shared memory");
 
 struct Bars {
-    uint64_t *q, *kv_full, *kv_empty, *s_full, *s_free, *sready, *o_done, *tail_s, *tail_o;
+    uint64_t *q, *k_full, *k_empty, *v_full, *v_empty, *s_full, *s_free, *sready, *o_done, *tail_s, *tail_o;
     uint32_t *tmem_slot;
     volatile int *abort_flag;
     __device__ Bars(uint8_t *base) {
         uint64_t *b = reinterpret_cast<uint64_t *>(base);
         q = b;
-        kv_full = b + 1;     // [2]
-        kv_empty = b + 3;    // [2]
-        s_full = b + 5;      // [2]
-        s_free = b + 7;      // [2]
-        sready = b + 9;      // [2]
-        o_done = b + 11;     // [2]
-        tail_s = b + 13;
-        tail_o = b + 14;
-        tmem_slot = reinterpret_cast<uint32_t *>(b + 15);
-        abort_flag = reinterpret_cast<volatile int *>(b + 16);
+        k_full = b + 1;      // [2]
+        k_empty = b + 3;     // [2]
+        v_full = b + 5;      // [2]
+        v_empty = b + 7;     // [2]
+        s_full = b + 9;      // [2]
+        s_free = b + 11;     // [2]
+        sready = b + 13;     // [2]
+        o_done = b + 15;     // [2]
+        tail_s = b + 17;
+        tail_o = b + 18;
+        tmem_slot = reinterpret_cast<uint32_t *>(b + 19);
+        abort_flag = reinterpret_cast<volatile int *>(b + 20);
     }
     __device__ void init() {
         mbar_init(q, 1);
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&kv_full[i], 1);
-            mbar_init(&kv_empty[i], 1);
+            mbar_init(&k_full[i], 1);
+            mbar_init(&k_empty[i], 1);
+            mbar_init(&v_full[i], 1);
+            mbar_init(&v_empty[i], 1);
             mbar_init(&s_full[i], 1);
             mbar_init(&s_free[i], kConv32 / 32);   // one arrival per converter warp
             mbar_init(&sready[i], kConv32 / 32);
@@ -631,7 +639,8 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sq = smem + Smem32::q_off;
-    uint8_t *skv = smem + Smem32::kv_off;
+    uint8_t *sk = smem + Smem32::k_off;
+    uint8_t *sv = smem + Smem32::v_off;
     uint8_t *ss = smem + Smem32::s_off;
     float *part = reinterpret_cast<float *>(smem + Smem32::part_off);
     Bars bar(smem + Smem32::bar_off);
@@ -668,27 +677,46 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
             mbar_expect_tx(bar.q, 2 * Smem32::Q_KQ);
             for (int kq = 0; kq < 2; ++kq)
                 tma_load_3d(sq + kq * Smem32::Q_KQ, &a.tm_q, bar.q, kq * 32, qt * kQTile, 2 * hd);
-            int issued = 0;
+            // K of block b waits for S of block b - 2 (V^T has a thread of
+            // its own, below)
+            int k_issued = 0;
             for (int b = 0; b < nkb; ++b) {
                 const int st = b & 1;
-                // the stage was last used by block b - 2, released after its O
-                if (b >= 2 && !mbar_wait(&bar.kv_empty[st], uint32_t(((b - 2) >> 1) & 1), bar.abort_flag, a.err))
+                if (b >= 2 && !mbar_wait(&bar.k_empty[st], uint32_t(((b - 2) >> 1) & 1), bar.abort_flag, a.err))
                     break;
-                uint8_t *dst = skv + st * Smem32::KV_STAGE;
-                const int key0 = key_begin + b * kKeys32;
-                mbar_expect_tx(&bar.kv_full[st], Smem32::KV_STAGE);
+                mbar_expect_tx(&bar.k_full[st], Smem32::K_STAGE);
                 for (int kq = 0; kq < 2; ++kq)
-                    tma_load_3d(dst + kq * Smem32::K_KQ, &a.tm_k, &bar.kv_full[st], kq * 32, key0, 2 * hd);
-                tma_load_3d(dst + 2 * Smem32::K_KQ, &a.tm_vt, &bar.kv_full[st], key0, 0, 2 * hd);
-                ++issued;
+                    tma_load_3d(sk + st * Smem32::K_STAGE + kq * Smem32::K_KQ, &a.tm_k, &bar.k_full[st], kq * 32,
+                                key_begin + b * kKeys32, 2 * hd);
+                ++k_issued;
             }
             if (*bar.abort_flag) {
                 // every copy already issued lands before shared memory goes
                 for (int st = 0; st < 2; ++st) {
-                    const int uses = issued / 2 + (st < issued % 2 ? 1 : 0);
-                    if (uses > 0) mbar_wait_drain(&bar.kv_full[st], uint32_t((uses - 1) & 1));
+                    const int ku = k_issued / 2 + (st < k_issued % 2 ? 1 : 0);
+                    if (ku > 0) mbar_wait_drain(&bar.k_full[st], uint32_t((ku - 1) & 1));
                 }
                 mbar_wait_drain(bar.q, 0);
+            }
+        }
+    } else if (warp == kVLoadWarp32) {
+        // ----------------------------------------------- TMA loads, V^T ring
+        // V^T of block b waits for O of block b - 2
+        if (lane == 0 && nkb > 0) {
+            int v_issued = 0;
+            for (int b = 0; b < nkb; ++b) {
+                const int st = b & 1;
+                if (b >= 2 && !mbar_wait(&bar.v_empty[st], uint32_t(((b - 2) >> 1) & 1), bar.abort_flag, a.err))
+                    break;
+                mbar_expect_tx(&bar.v_full[st], Smem32::VT);
+                tma_load_3d(sv + st * Smem32::VT, &a.tm_vt, &bar.v_full[st], key_begin + b * kKeys32, 0, 2 * hd);
+                ++v_issued;
+            }
+            if (*bar.abort_flag) {
+                for (int st = 0; st < 2; ++st) {
+                    const int vu = v_issued / 2 + (st < v_issued % 2 ? 1 : 0);
+                    if (vu > 0) mbar_wait_drain(&bar.v_full[st], uint32_t((vu - 1) & 1));
+                }
             }
         }
     } else if (warp == kSWarp32) {
@@ -698,13 +726,13 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
             const uint32_t qa = smem_addr(sq);
             for (int b = 0; ok && b < nkb; ++b) {
                 const int st = b & 1;
-                if (!mbar_wait(&bar.kv_full[st], uint32_t((b >> 1) & 1), bar.abort_flag, a.err) ||
+                if (!mbar_wait(&bar.k_full[st], uint32_t((b >> 1) & 1), bar.abort_flag, a.err) ||
                     (b >= 2 && !mbar_wait(&bar.s_free[st], uint32_t(((b - 2) >> 1) & 1), bar.abort_flag, a.err))) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t ka = smem_addr(skv + st * Smem32::KV_STAGE);
+                const uint32_t ka = smem_addr(sk + st * Smem32::K_STAGE);
                 const uint32_t tS = tmem + kTmemS + uint32_t(st * 2 * kKeys32);
                 for (int kq = 0; kq < 2; ++kq)
 #pragma unroll
@@ -715,6 +743,7 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
                         mma_tf32(tS, make_sdesc(qb + kQTile * 128), kd, kIdescS32First, 1u);
                     }
                 tc_commit(&bar.s_full[st]);
+                tc_commit(&bar.k_empty[st]);
             }
             if (!ok) {
                 tc_commit(bar.tail_s);
@@ -726,12 +755,13 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
         if (lane == 0 && nkb > 0) {
             for (int b = 0; ok && b < nkb; ++b) {
                 const int st = b & 1;
-                if (!mbar_wait(&bar.sready[st], uint32_t((b >> 1) & 1), bar.abort_flag, a.err)) {
+                if (!mbar_wait(&bar.sready[st], uint32_t((b >> 1) & 1), bar.abort_flag, a.err) ||
+                    !mbar_wait(&bar.v_full[st], uint32_t((b >> 1) & 1), bar.abort_flag, a.err)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t va = smem_addr(skv + st * Smem32::KV_STAGE) + 2 * Smem32::K_KQ;
+                const uint32_t va = smem_addr(sv + st * Smem32::VT);
                 const uint32_t sa = smem_addr(ss + st * Smem32::S);
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
@@ -739,9 +769,8 @@ __global__ void __launch_bounds__(attn::kThreads32, 1)
                     mma_tf32(tO, make_sdesc(va + kk * 32), sd, kIdescO32, (b > 0 || kk > 0) ? 1u : 0u);
                     mma_tf32(tO, make_sdesc(va + 128 * 128 + kk * 32), sd, kIdescO32First, 1u);
                 }
-                // S_b finished before it was split, so this also frees K
                 tc_commit(&bar.o_done[st]);
-                tc_commit(&bar.kv_empty[st]);
+                tc_commit(&bar.v_empty[st]);
             }
             if (!ok) {
                 tc_commit(bar.tail_o);
