@@ -537,6 +537,7 @@ static qx_status build_gemm(qx_plan p) {
     a.m_extent = int(d.N);
     a.n_extent = int(d.M);
     a.kblocks = int((d.K + kBK - 1) / kBK);
+    a.k_valid = int(d.K);
     a.chunk_kb = int(s.chunk_kb);
     a.tiles_m = int((d.N + kBM - 1) / kBM);
     a.tiles_n = int((d.M + mr - 1) / mr);
@@ -680,6 +681,7 @@ static qx_status build_conv_patches(qx_plan p) {
     a.m_extent = int(M);
     a.n_extent = int(d.k_out);
     a.kblocks = int((p->Kp + kBK - 1) / kBK);
+    a.k_valid = int(p->Kp);
     a.chunk_kb = int(s.chunk_kb);
     a.tiles_m = int((M + kBM - 1) / kBM);
     a.tiles_n = int((d.k_out + mr - 1) / mr);

@@ -63,6 +63,11 @@ struct MmaArgs {
     int chunk_kb;             // k-blocks per FP32 accumulation chunk
     int tiles_m, tiles_n, group_n;
     int mr;                   // N-side rows per limb of the tile (128 or 64)
+    int k_valid;              // K elements holding data (0: every k-block full); the
+                              // tensor-core sub-steps of the last k-block past it are skipped
+    // set by the launcher from the two fields above and the kernel instance
+    int k_tail_steps;         // 16-wide K sub-steps issued in the last k-block (1..4)
+    int n_resident;           // one N-side tile: its k-blocks are loaded once per CTA
     int shift_n, shift_m;     // digit widths of the N-side / M-side limbs
     // conv geometry (modes 1 and 2)
     int c_blocks, S, Q, PQ, stride, pad, k_out;

@@ -36,6 +36,8 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <type_traits>
+
 #include "qx_device.cuh"
 #include "qx_internal.h"
 #include "qx_tile.cuh"
@@ -51,9 +53,10 @@ __global__ void __launch_bounds__(384, 1) limb_gemm_kernel(const __grid_constant
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + T::STAGES * T::STAGE);
     uint64_t *empty = full + T::STAGES;
     uint64_t *acc_full = empty + T::STAGES;
-    uint64_t *acc_empty = acc_full + 2;
-    uint64_t *tail = acc_empty + 2;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(tail + 1);
+    uint64_t *acc_empty = acc_full + T::ACC_BUFS;
+    uint64_t *tail = acc_empty + T::ACC_BUFS;
+    uint64_t *n_loaded = tail + 1;      // resident N-side tile landed
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(n_loaded + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
@@ -67,14 +70,16 @@ __global__ void __launch_bounds__(384, 1) limb_gemm_kernel(const __grid_constant
         if (NB > 1) tma_prefetch(&a.tm_m[1]);
         tma_prefetch(&a.tm_n);
         for (int s = 0; s < T::STAGES; ++s) {
-            mbar_init(&full[s], 2);          // one arrive.expect_tx per producer
+            // one arrive.expect_tx per producer whose loads go through the ring
+            mbar_init(&full[s], a.n_resident ? 1 : 2);
             mbar_init(&empty[s], 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < T::ACC_BUFS; ++b) {
             mbar_init(&acc_full[b], 1);
             mbar_init(&acc_empty[b], 8);
         }
         mbar_init(tail, 1);
+        mbar_init(n_loaded, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -162,53 +167,71 @@ __global__ void __launch_bounds__(384, 1) limb_gemm_kernel(const __grid_constant
             int stage = 0;
             uint32_t phase = 0;
             uint32_t acc_it = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
-                for (int kb0 = 0; kb0 < a.kblocks; kb0 += a.chunk_kb) {
-                    const int kb1 = min(kb0 + a.chunk_kb, a.kblocks);
-                    const uint32_t buf = T::NBUF == 2 ? (acc_it & 1u) : 0u;
-                    const uint32_t apar = T::NBUF == 2 ? ((acc_it >> 1) & 1u) : (acc_it & 1u);
-                    if (!mbar_wait(&acc_empty[buf], apar ^ 1, abort_flag, a.err)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint32_t d0 = tmem_base + buf * T::ACC_COLS;
-                    for (int kb = kb0; kb < kb1; ++kb) {
-                        if (!mbar_wait(&full[stage], phase, abort_flag, a.err)) {
-                            ok = false;
-                            break;
-                        }
+            // The issue loop is this thread's critical path on large problems
+            // (a few hundred cycles per k-block): its variants are compiled
+            // separately so that the common one does no per-k-block work for
+            // a resident N-side tile (RES) or a short last k-block (TAIL).
+            auto issue_all = [&](auto res_c, auto tail_c) -> bool {
+                constexpr bool RES = decltype(res_c)::value;
+                constexpr bool TAIL = decltype(tail_c)::value;
+                for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
+                    for (int kb0 = 0; kb0 < a.kblocks; kb0 += a.chunk_kb) {
+                        const int kb1 = min(kb0 + a.chunk_kb, a.kblocks);
+                        const uint32_t buf = acc_it % T::ACC_BUFS;
+                        const uint32_t apar = (acc_it / T::ACC_BUFS) & 1u;
+                        if (!mbar_wait(&acc_empty[buf], apar ^ 1, abort_flag, a.err)) return false;
                         tc_fence_after();
-                        const uint32_t sbase = smem_addr(smem + stage * T::STAGE);
+                        const uint32_t d0 = tmem_base + buf * T::ACC_COLS;
+                        for (int kb = kb0; kb < kb1; ++kb) {
+                            if (!mbar_wait(&full[stage], phase, abort_flag, a.err)) return false;
+                            tc_fence_after();
+                            const uint32_t sbase = smem_addr(smem + stage * T::STAGE);
+                            // N-side tile: this stage's, or the resident copy of k-block kb
+                            const uint32_t nbase =
+                                (RES ? smem_addr(smem + kb * T::STAGE) : sbase) + NB * T::M_TILE;
+                            // sub-steps wholly past the data multiply zeros: skip them
+                            const int nk = TAIL && kb == a.kblocks - 1 ? a.k_tail_steps : 4;
 #pragma unroll
-                        for (int kk = 0; kk < 4; ++kk) {          // 4 x 32 bytes of K per row
-                            const uint64_t bdesc = make_sdesc(sbase + NB * T::M_TILE + kk * 32);
-                            const uint32_t acc = (kb > kb0 || kk > 0) ? 1u : 0u;
-                            if constexpr (T::TF) {
-                                // x_big * [w_big; w_small], then x_small * w_big
-                                mma_tf32(d0, make_sdesc(sbase + kk * 32), bdesc, T::IDESC, acc);
-                                mma_tf32(d0, make_sdesc(sbase + T::M_TILE + kk * 32), bdesc,
-                                         T::IDESC_FIRST, 1u);
-                            } else {
+                            for (int kk = 0; kk < 4; ++kk) {          // 4 x 32 bytes of K per row
+                                if (TAIL && kk >= nk) break;
+                                const uint64_t bdesc = make_sdesc(nbase + kk * 32);
+                                const uint32_t acc = (kb > kb0 || kk > 0) ? 1u : 0u;
+                                if constexpr (T::TF) {
+                                    // x_big * [w_big; w_small], then x_small * w_big
+                                    mma_tf32(d0, make_sdesc(sbase + kk * 32), bdesc, T::IDESC, acc);
+                                    mma_tf32(d0, make_sdesc(sbase + T::M_TILE + kk * 32), bdesc,
+                                             T::IDESC_FIRST, 1u);
+                                } else {
 #pragma unroll
-                                for (int j = 0; j < NB; ++j) {
-                                    const uint64_t adesc =
-                                        make_sdesc(sbase + j * T::M_TILE + kk * 32);
-                                    mma_f16(d0 + j * T::UN, adesc, bdesc, T::IDESC, acc);
+                                    for (int j = 0; j < NB; ++j) {
+                                        const uint64_t adesc =
+                                            make_sdesc(sbase + j * T::M_TILE + kk * 32);
+                                        mma_f16(d0 + j * T::UN, adesc, bdesc, T::IDESC, acc);
+                                    }
                                 }
                             }
+                            tc_commit(&empty[stage]);
+                            if (++stage == T::STAGES) {
+                                stage = 0;
+                                phase ^= 1;
+                            }
                         }
-                        tc_commit(&empty[stage]);
-                        if (++stage == T::STAGES) {
-                            stage = 0;
-                            phase ^= 1;
-                        }
+                        tc_commit(&acc_full[buf]);
+                        ++acc_it;
                     }
-                    if (!ok) break;
-                    tc_commit(&acc_full[buf]);
-                    ++acc_it;
                 }
+                return true;
+            };
+            using yes = std::true_type;
+            using no = std::false_type;
+            bool ok = true;
+            if (a.n_resident) ok = mbar_wait(n_loaded, 0, abort_flag, a.err);
+            if (ok) {
+                const bool tail = !T::TF && a.k_tail_steps < 4;
+                if (a.n_resident)
+                    ok = tail ? issue_all(yes{}, yes{}) : issue_all(yes{}, no{});
+                else
+                    ok = tail ? issue_all(no{}, yes{}) : issue_all(no{}, no{});
             }
             if (!ok) {
                 // MMAs already issued must finish before TMEM is released.
@@ -219,33 +242,45 @@ __global__ void __launch_bounds__(384, 1) limb_gemm_kernel(const __grid_constant
     } else if (warp == T::N_PRODUCER_WARP) {
         if (lane == 0) {
             // ---------------------------------------- TMA producer, N side
-            int stage = 0;
-            uint32_t phase = 0;
-            long long issued = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
-                int tm, tn;
-                tile_coords(t, a, tm, tn);
-                for (int kb = 0; kb < a.kblocks; ++kb) {
-                    if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, a.err)) {
-                        ok = false;
-                        break;
-                    }
-                    mbar_expect_tx(&full[stage], T::N_TILE);
-                    tma_load_3d(smem + stage * T::STAGE + NB * T::M_TILE, &a.tm_n, &full[stage],
-                                kb * T::BK_ELEMS, tn * T::MR, 0);
-                    ++issued;
-                    if (++stage == T::STAGES) {
-                        stage = 0;
-                        phase ^= 1;
+            if (a.n_resident) {
+                // The only N-side tile, every k-block of it, once per CTA:
+                // k-block kb goes to the N part of stage kb's buffer, which
+                // the ring leaves alone in this mode.  The copies must land
+                // before shared memory goes, whatever else happens.
+                mbar_expect_tx(n_loaded, uint32_t(a.kblocks) * T::N_TILE);
+                for (int kb = 0; kb < a.kblocks; ++kb)
+                    tma_load_3d(smem + kb * T::STAGE + NB * T::M_TILE, &a.tm_n, n_loaded,
+                                kb * T::BK_ELEMS, 0, 0);
+                mbar_wait_drain(n_loaded, 0);
+            } else {
+                int stage = 0;
+                uint32_t phase = 0;
+                long long issued = 0;
+                bool ok = true;
+                for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+                    int tm, tn;
+                    tile_coords(t, a, tm, tn);
+                    for (int kb = 0; kb < a.kblocks; ++kb) {
+                        if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, a.err)) {
+                            ok = false;
+                            break;
+                        }
+                        mbar_expect_tx(&full[stage], T::N_TILE);
+                        tma_load_3d(smem + stage * T::STAGE + NB * T::M_TILE, &a.tm_n, &full[stage],
+                                    kb * T::BK_ELEMS, tn * T::MR, 0);
+                        ++issued;
+                        if (++stage == T::STAGES) {
+                            stage = 0;
+                            phase ^= 1;
+                        }
                     }
                 }
-            }
-            if (*abort_flag) {
-                // Let every copy already issued land before shared memory goes.
-                for (int s = 0; s < T::STAGES; ++s) {
-                    const long long uses = issued / T::STAGES + (s < issued % T::STAGES ? 1 : 0);
-                    if (uses > 0) mbar_wait_drain(&full[s], uint32_t((uses - 1) & 1));
+                if (*abort_flag) {
+                    // Let every copy already issued land before shared memory goes.
+                    for (int s = 0; s < T::STAGES; ++s) {
+                        const long long uses = issued / T::STAGES + (s < issued % T::STAGES ? 1 : 0);
+                        if (uses > 0) mbar_wait_drain(&full[s], uint32_t((uses - 1) & 1));
+                    }
                 }
             }
         }
@@ -263,8 +298,8 @@ __global__ void __launch_bounds__(384, 1) limb_gemm_kernel(const __grid_constant
 #pragma unroll
             for (int r = 0; r < T::RPT; ++r) acc[r] = 0u;
             for (int kb0 = 0; kb0 < a.kblocks; kb0 += a.chunk_kb) {
-                const uint32_t buf = T::NBUF == 2 ? (acc_it & 1u) : 0u;
-                const uint32_t apar = T::NBUF == 2 ? ((acc_it >> 1) & 1u) : (acc_it & 1u);
+                const uint32_t buf = acc_it % T::ACC_BUFS;
+                const uint32_t apar = (acc_it / T::ACC_BUFS) & 1u;
                 if (!mbar_wait(&acc_full[buf], apar, abort_flag, a.err)) {
                     ok = false;
                     break;
@@ -316,9 +351,20 @@ static cudaError_t prepare_t() {
                                 TileCfg<NA, NB, KIND, MR_>::SMEM);
 }
 
+// The launch-time fields: how many K sub-steps the last k-block issues, and
+// whether the N-side operand is one tile whose k-blocks all fit in the stage
+// buffers (then it is loaded once per CTA instead of once per output tile:
+// every CTA would otherwise re-read the same few L2 lines for every tile).
 template <int NA, int NB, int KIND = kKindExact, int MR_ = TileCfg<NA, NB, KIND>::MR>
-static cudaError_t launch_t(const MmaArgs &a, int grid, cudaStream_t stream) {
+static cudaError_t launch_t(const MmaArgs &a0, int grid, cudaStream_t stream) {
     using T = TileCfg<NA, NB, KIND, MR_>;
+    MmaArgs a = a0;
+    a.k_tail_steps = 4;
+    if (!T::TF && a.k_valid > 0) {
+        const int rem = a.k_valid - (a.kblocks - 1) * kBK;
+        if (rem > 0 && rem < kBK) a.k_tail_steps = (rem + 15) / 16;
+    }
+    a.n_resident = (a.tiles_n == 1 && a.kblocks >= 1 && a.kblocks <= T::STAGES) ? 1 : 0;
     return launch_pdl(limb_gemm_kernel<NA, NB, KIND, MR_>, grid, T::THREADS, T::SMEM, stream, a);
 }
 

@@ -278,6 +278,7 @@ extern "C" qx_status qx_gemm_i16_i32_noalloc(int64_t M, int64_t N, int64_t K, qx
     a.m_extent = int(N);
     a.n_extent = int(M);
     a.kblocks = int((K + kBK - 1) / kBK);
+    a.k_valid = int(K);
     a.chunk_kb = int(s.chunk_kb);
     a.tiles_m = int((N + kBM - 1) / kBM);
     a.tiles_n = int((M + mr - 1) / mr);

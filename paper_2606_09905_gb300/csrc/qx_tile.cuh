@@ -25,7 +25,12 @@ struct TileCfg {
     // exact kind; the TF32 kind sums all products into one.
     static constexpr int ACC_COLS = TF ? UN : NB * UN;
     static constexpr int NBUF = ACC_COLS <= 256 ? 2 : 1;
-    static constexpr int TMEM_NEED = ACC_COLS * NBUF;
+    // Accumulator sets of the limb kernel: four when they fit in half of
+    // TMEM, so that the MMAs of short tiles (one or two k-blocks) run up to
+    // three tiles ahead of the epilogue instead of waiting for the round trip
+    // commit -> drain -> release of the set before last.
+    static constexpr int ACC_BUFS = ACC_COLS <= 128 ? 4 : NBUF;
+    static constexpr int TMEM_NEED = ACC_COLS * ACC_BUFS;
     static constexpr int TMEM_COLS = TMEM_NEED <= 32    ? 32
                                      : TMEM_NEED <= 64  ? 64
                                      : TMEM_NEED <= 128 ? 128
@@ -47,6 +52,8 @@ struct TileCfg {
     static constexpr int M_PRODUCER2_WARP = 11;
     static_assert(UN % 16 == 0 && UN >= 16 && UN <= 256, "MMA N out of range");
     static_assert(TMEM_NEED <= 512, "accumulators exceed tensor memory");
+    static_assert((2 * STAGES + 2 * ACC_BUFS + 2) * 8 + 8 <= BAR_BYTES, "barriers exceed their area");
+    static_assert(SMEM <= 232448, "shared memory over the per-CTA limit");
     static_assert(RPT % 32 == 0, "epilogue works in 32-column TMEM loads");
     static_assert(!TF || (NA == 2 && NB == 2), "TF32x3 stacks big/small on both sides");
 };
@@ -67,7 +74,9 @@ __device__ __forceinline__ void tile_coords(int t, const MmaArgs &a, int &tm, in
 // Exact kind: add one chunk's accumulators (every M-side limb j, N-side limb
 // i) into the running wrapping int32 sums of this thread.  `tb` addresses the
 // thread's TMEM lane quarter, the accumulator set and its half of the N-side
-// rows; 32-row groups wholly past the N-side extent are skipped.
+// rows; 32-row groups wholly past the N-side extent are skipped, and a group
+// with at most 8 rows inside it reads 8 columns instead of 32 (narrow
+// outputs: the 6 output channels of a LeNet conv1, the 10 logits of its fc3).
 template <int NA, int NB, int MR_>
 __device__ __forceinline__ void drain_exact(uint32_t tb, int rows_left, int shift_n, int shift_m,
                                             uint32_t (&acc)[TileCfg<NA, NB, kKindExact, MR_>::RPT]) {
@@ -79,13 +88,24 @@ __device__ __forceinline__ void drain_exact(uint32_t tb, int rows_left, int shif
             const int sh = i * shift_n + j * shift_m;
 #pragma unroll
             for (int p = 0; p < T::RPT / 32; ++p) {
-                if (p * 32 >= rows_left) continue;
-                uint32_t v[32];
-                tmem_ld32(tb + j * T::UN + i * T::MR + p * 32, v);
-                tmem_wait_ld(v);
+                const int w = rows_left - p * 32;
+                if (w <= 0) continue;
+                const uint32_t col = tb + j * T::UN + i * T::MR + p * 32;
+                if (w <= 8) {
+                    uint32_t v[8];
+                    tmem_ld8(col, v);
+                    tmem_wait_ld8(v);
 #pragma unroll
-                for (int x = 0; x < 32; ++x)
-                    acc[p * 32 + x] += uint32_t(__float2int_rn(__uint_as_float(v[x]))) << sh;
+                    for (int x = 0; x < 8; ++x)
+                        acc[p * 32 + x] += uint32_t(__float2int_rn(__uint_as_float(v[x]))) << sh;
+                } else {
+                    uint32_t v[32];
+                    tmem_ld32(col, v);
+                    tmem_wait_ld(v);
+#pragma unroll
+                    for (int x = 0; x < 32; ++x)
+                        acc[p * 32 + x] += uint32_t(__float2int_rn(__uint_as_float(v[x]))) << sh;
+                }
             }
         }
     }
@@ -93,13 +113,18 @@ __device__ __forceinline__ void drain_exact(uint32_t tb, int rows_left, int shif
 
 // Store a finished tile: this thread owns output column (M-side row)
 // tm*128 + q*32 + lane and N-side rows nrow0 .. nrow0 + RPT - 1.  Conv modes
-// write NCHW.  Integer kinds apply the optional ReLU-requantize first.
+// write NCHW.  Integer kinds apply the optional ReLU-requantize first.  Work
+// stops at the N-side extent, one 32-row group at a time, so a narrow output
+// costs its valid rows only.  (Staging the rows in shared memory for 16-byte
+// stores was measured slower, for narrow and wide outputs alike.)
 template <int NA, int NB, int KIND, int MR_>
 __device__ __forceinline__ void store_tile(const MmaArgs &a, int tm, int tn, int q, int hh, int lane,
                                            uint32_t (&acc)[TileCfg<NA, NB, KIND, MR_>::RPT]) {
     using T = TileCfg<NA, NB, KIND, MR_>;
+    const int nrow0 = tn * T::MR + hh * T::RPT;
+    const int rows = a.n_extent - nrow0;
     const int mrow = tm * kBM + q * 32 + lane;
-    const bool lane_ok = mrow < a.m_extent;
+    if (rows <= 0 || mrow >= a.m_extent) return;
     int64_t lane_off = mrow;
     if (a.mode != 0) {   // conv: pixel mrow of image img, NCHW output
         const int img = mrow / a.PQ;
@@ -112,12 +137,16 @@ __device__ __forceinline__ void store_tile(const MmaArgs &a, int tm, int tn, int
                 acc[r] = uint32_t(min(max(int32_t(acc[r]), 0) >> a.rq_shift, a.rq_hi));
         }
     }
-    const int nrow0 = tn * T::MR + hh * T::RPT;
     // both output types are 32-bit: store the raw words
     uint32_t *o = static_cast<uint32_t *>(a.out) + lane_off + int64_t(nrow0) * a.out_row_stride;
 #pragma unroll
-    for (int r = 0; r < T::RPT; ++r) {
-        if (lane_ok && nrow0 + r < a.n_extent) o[int64_t(r) * a.out_row_stride] = acc[r];
+    for (int p = 0; p < T::RPT / 32; ++p) {
+        if (p * 32 >= rows) break;
+#pragma unroll
+        for (int x = 0; x < 32; ++x) {
+            const int r = p * 32 + x;
+            if (r < rows) o[int64_t(r) * a.out_row_stride] = acc[r];
+        }
     }
 }
 
