@@ -36,6 +36,19 @@ struct RangeCheck {
     }
 };
 
+// Digits to FP16, two at a time: a digit d (|d| <= 2048 under the contract)
+// becomes an exact float by the 1.5 * 2^23 bit-pattern trick (the float with
+// bits 0x4B400000 + d is 1.5 * 2^23 + d for |d| < 2^22; one integer add and
+// one float subtract, both full-rate), and each pair is rounded to a half2 by
+// one conversion -- half the conversion-pipe work of one int -> half
+// conversion per digit.
+__device__ __forceinline__ uint32_t digits_to_half2(int32_t d0, int32_t d1) {
+    const float f0 = __int_as_float(0x4B400000 + d0) - 12582912.0f;
+    const float f1 = __int_as_float(0x4B400000 + d1) - 12582912.0f;
+    const __half2 h = __floats2half2_rn(f0, f1);     // f0 in the low half
+    return *reinterpret_cast<const uint32_t *>(&h);
+}
+
 template <int NL>
 __device__ __forceinline__ void store_limbs8(__half *plane0, int64_t plane_stride, const int32_t (&v)[8],
                                              int shift) {
@@ -44,10 +57,12 @@ __device__ __forceinline__ void store_limbs8(__half *plane0, int64_t plane_strid
     for (int e = 0; e < 8; ++e) split_digits<NL>(v[e], shift, d[e]);
 #pragma unroll
     for (int i = 0; i < NL; ++i) {
-        __align__(16) __half h[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) h[e] = __int2half_rn(d[e][i]);
-        *reinterpret_cast<uint4 *>(plane0 + i * plane_stride) = *reinterpret_cast<uint4 *>(h);
+        uint4 w;
+        w.x = digits_to_half2(d[0][i], d[1][i]);
+        w.y = digits_to_half2(d[2][i], d[3][i]);
+        w.z = digits_to_half2(d[4][i], d[5][i]);
+        w.w = digits_to_half2(d[6][i], d[7][i]);
+        *reinterpret_cast<uint4 *>(plane0 + i * plane_stride) = w;
     }
 }
 
@@ -327,6 +342,150 @@ __global__ void __launch_bounds__(256) pack_patches_kernel(const PatchPackArgs p
         }
         p.cw.test8(v, RSC - 8 * g, p.err);
         store_limbs8<NW>(p.w_planes + int64_t(o) * p.Kp + 8 * g, plane_stride, v, p.shift_w);
+    }
+}
+
+// Division by a divisor fixed for the launch, as a multiply and a shift
+// (Granlund and Montgomery, "Division by invariant integers using
+// multiplication", PLDI 1994, Theorem 4.2 with N = 31): with
+// l = ceil(log2 d) and m = ceil(2^(31+l) / d), m d - 2^(31+l) < d <= 2^l, so
+// floor(n / d) = floor(m n / 2^(31+l)) for every 0 <= n < 2^31.
+struct InvDiv {
+    uint32_t m;
+    int sh;
+    __device__ __forceinline__ int div(int n) const {
+        return int((uint64_t(uint32_t(n)) * m) >> sh);
+    }
+};
+
+static InvDiv make_invdiv(int d) {
+    int l = 0;
+    while ((int64_t(1) << l) < d) ++l;
+    const uint64_t two = uint64_t(1) << (31 + l);
+    InvDiv v;
+    v.m = uint32_t((two + uint64_t(d) - 1) / uint64_t(d));
+    v.sh = 31 + l;
+    return v;
+}
+
+// x side of the patch lowering, one image at a time: the image, zero-padded
+// by `pad` on every side, is staged in shared memory with coalesced loads,
+// and every patch element is then one shared-memory read at the window
+// corner plus a tabled offset -- no bounds tests, no per-element global
+// gathers.  Used when the padded image and the offset table fit in 48 KB
+// (the small-channel convs this lowering serves: LeNet's conv1 reads a
+// 4 KB image, its conv2 a 4.7 KB one).  Every in-bounds value is checked
+// against the range contract when it is staged.  Blocks past `x_blocks`
+// lower the weights exactly as pack_patches_kernel does.
+struct PatchImgArgs {
+    PatchPackArgs p;
+    InvDiv by_groups, by_q, by_hwp, by_wp;
+};
+
+template <typename T, int NX, int NW>
+__global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArgs pa) {
+    pdl_launch_dependents();
+    const PatchPackArgs &p = pa.p;
+    extern __shared__ int32_t psm[];
+    const int Kp = p.Kp;
+    int32_t *koff = psm;                                  // Kp entries, -1 past c r s
+    int32_t *img = psm + ((Kp + 3) & ~3);
+    const int hp = p.h + 2 * p.pad, wp = p.wd + 2 * p.pad;
+    const int HWp = hp * wp;
+    const int RSC = p.r * p.s * p.c;
+    const int groups = Kp >> 3;
+    if (int(blockIdx.x) >= p.x_blocks) {
+        const T *W = static_cast<const T *>(p.w);
+        const int64_t items = int64_t(p.k_out) * groups;
+        const int64_t plane_stride = int64_t(p.k_out) * Kp;
+        const int RS = p.r * p.s;
+        for (int64_t it = int64_t(blockIdx.x - p.x_blocks) * blockDim.x + threadIdx.x; it < items;
+             it += int64_t(gridDim.x - p.x_blocks) * blockDim.x) {
+            const int o = int(it / groups);
+            const int g = int(it - int64_t(o) * groups);
+            int32_t v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int k = 8 * g + e;
+                const int tap = k / p.c;
+                const int ch = k - tap * p.c;
+                v[e] = k < RSC ? int32_t(W[(int64_t(o) * p.c + ch) * RS + tap]) : 0;
+            }
+            p.cw.test8(v, RSC - 8 * g, p.err);
+            store_limbs8<NW>(p.w_planes + int64_t(o) * Kp + 8 * g, plane_stride, v, p.shift_w);
+        }
+        return;
+    }
+    for (int k = threadIdx.x; k < Kp; k += blockDim.x) {
+        int32_t off = -1;
+        if (k < RSC) {
+            const int tap = k / p.c;
+            const int ch = k - tap * p.c;
+            const int rr = tap / p.s;
+            off = ch * HWp + rr * wp + (tap - rr * p.s);
+        }
+        koff[k] = off;
+    }
+    const T *X = static_cast<const T *>(p.x);
+    const int HW = p.h * p.wd;
+    const int PQ = p.P * p.Q;
+    const int items = PQ * groups;                        // < 2^31 (the launcher checks)
+    const int64_t plane_stride = int64_t(p.n) * PQ * Kp;
+    const int CHWp = p.c * HWp;
+    const bool fixed_g = int(blockDim.x) % groups == 0;
+    const int pix0 = pa.by_groups.div(threadIdx.x);       // first pixel of this thread
+    const int gsel = int(threadIdx.x) - pix0 * groups;    // its group of 8 elements
+    const int pix_step = int(blockDim.x) / groups;
+    int32_t off8[8];
+    __syncthreads();                                      // koff is complete
+#pragma unroll
+    for (int e = 0; e < 8; ++e) off8[e] = fixed_g ? koff[8 * gsel + e] : -1;
+    for (int im = blockIdx.x; im < p.n; im += p.x_blocks) {
+        __syncthreads();                                  // the previous image is consumed
+        const T *xs = X + int64_t(im) * p.c * HW;
+        for (int i = threadIdx.x; i < CHWp; i += blockDim.x) {
+            const int ch = pa.by_hwp.div(i);
+            const int rem = i - ch * HWp;
+            const int y = pa.by_wp.div(rem);
+            const int iy = y - p.pad;
+            const int ix = rem - y * wp - p.pad;
+            int32_t v = 0;
+            if (unsigned(iy) < unsigned(p.h) && unsigned(ix) < unsigned(p.wd)) {
+                v = int32_t(xs[ch * HW + iy * p.wd + ix]);
+                p.cx.test(v, p.err);
+            }
+            img[i] = v;
+        }
+        __syncthreads();
+        __half *dst = p.x_planes + int64_t(im) * PQ * Kp;
+        if (fixed_g) {
+            // the block is a whole number of pixels wide: this thread keeps
+            // its group and its eight offsets for the whole image
+            for (int pix = pix0; pix < PQ; pix += pix_step) {
+                const int oh = pa.by_q.div(pix);
+                const int ow = pix - oh * p.Q;
+                const int32_t *corner = img + oh * p.stride * wp + ow * p.stride;
+                int32_t v[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) v[e] = off8[e] >= 0 ? corner[off8[e]] : 0;
+                store_limbs8<NX>(dst + int64_t(pix) * Kp + 8 * gsel, plane_stride, v, p.shift_x);
+            }
+            continue;
+        }
+        for (int it = threadIdx.x; it < items; it += blockDim.x) {
+            const int pix = pa.by_groups.div(it);
+            const int g = it - pix * groups;
+            const int oh = pa.by_q.div(pix);
+            const int ow = pix - oh * p.Q;
+            const int32_t *corner = img + oh * p.stride * wp + ow * p.stride;
+            int32_t v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int off = koff[8 * g + e];
+                v[e] = off >= 0 ? corner[off] : 0;
+            }
+            store_limbs8<NX>(dst + int64_t(pix) * Kp + 8 * g, plane_stride, v, p.shift_x);
+        }
     }
 }
 
@@ -650,6 +809,19 @@ static cudaError_t pack_patches_t(int nx, int nw, const PatchPackArgs &p, int gr
     return cudaErrorInvalidValue;
 }
 
+template <typename T>
+static cudaError_t pack_patches_img_t(int nx, int nw, const PatchImgArgs &pa, int grid, int threads,
+                                      int smem, cudaStream_t st) {
+#define QX_PPI(A_, B_)                                                                 \
+    if (nx == A_ && nw == B_) {                                                        \
+        pack_patches_img_kernel<T, A_, B_><<<grid, threads, smem, st>>>(pa);           \
+        return cudaGetLastError();                                                     \
+    }
+    QX_PPI(1, 1) QX_PPI(1, 2) QX_PPI(1, 3) QX_PPI(1, 4) QX_PPI(2, 1) QX_PPI(2, 2) QX_PPI(2, 4)
+#undef QX_PPI
+    return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_pack_patches(bool i32, const void *x, const void *w, int n, int c, int h, int wd,
                                 int k_out, int r, int s, int stride, int pad, int P, int Q, int Kp,
                                 __half *x_planes, __half *w_planes, int nx, int shift_x, int nw,
@@ -685,6 +857,24 @@ cudaError_t launch_pack_patches(bool i32, const void *x, const void *w, int n, i
     int w_blocks = int((w_items + 255) / 256);
     if (w_blocks > num_sms) w_blocks = num_sms;
     if (w_blocks < 1) w_blocks = 1;
+    // one image at a time through shared memory when it fits
+    const int64_t hp = int64_t(h) + 2 * pad, wp = int64_t(wd) + 2 * pad;
+    const int64_t img_words = int64_t(c) * hp * wp;
+    const int64_t smem = (((int64_t(Kp) + 3) & ~int64_t(3)) + img_words) * 4;
+    if (smem <= 48 * 1024 && int64_t(P) * Q * (Kp / 8) < (int64_t(1) << 31)) {
+        PatchImgArgs pa;
+        pa.p = p;
+        pa.p.x_blocks = n < num_sms * 8 ? n : num_sms * 8;
+        pa.by_groups = make_invdiv(Kp / 8);
+        pa.by_q = make_invdiv(Q);
+        pa.by_hwp = make_invdiv(int(hp * wp));
+        pa.by_wp = make_invdiv(int(wp));
+        const int grid = pa.p.x_blocks + w_blocks;
+        const int groups = Kp / 8;
+        const int threads = groups <= 256 ? groups * (256 / groups) : 256;
+        return i32 ? pack_patches_img_t<int32_t>(nx, nw, pa, grid, threads, int(smem), st)
+                   : pack_patches_img_t<int16_t>(nx, nw, pa, grid, threads, int(smem), st);
+    }
     return i32 ? pack_patches_t<int32_t>(nx, nw, p, p.x_blocks + w_blocks, st)
                : pack_patches_t<int16_t>(nx, nw, p, p.x_blocks + w_blocks, st);
 }

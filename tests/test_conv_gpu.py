@@ -154,6 +154,9 @@ def test_conv_f32_integer_values_exact():
     ((64, 6, 14, 14, 16, 5, 5), 1, 0),        # LeNet conv2
     ((3, 31, 9, 9, 33, 3, 3), 1, 1),
     ((2, 2, 11, 7, 130, 3, 2), 2, 1),
+    ((3, 3, 10, 13, 8, 5, 5), 1, 2),          # halo wider than one tap
+    ((2, 16, 60, 60, 24, 3, 3), 1, 1),        # image too large to stage: gather path
+    ((1, 4, 9, 9, 7, 4, 2), 3, 0),            # stride 3: unused edge rows and columns
 ])
 def test_conv_explicit_patches(shape, stride, pad):
     n, c, h, wd, k, r, s = shape
@@ -162,6 +165,25 @@ def test_conv_explicit_patches(shape, stride, pad):
     got, st, info = conv_gpu(x, w, stride, pad, (-255, 255), (-255, 255), dtype=qx.I32)
     assert st == qx.OK
     assert_exact(got, ref, f"conv {shape} s{stride} p{pad} {info}")
+
+
+@pytest.mark.parametrize("h", [14, 60])   # staged image, gather path
+def test_conv_explicit_patches_range_check(h):
+    x, w = inputs.conv_case(2, 6, h, h, 16, 5, 5, 0, 255, seed=h, dtype=torch.int32)
+    x[1, 3, h // 2, h // 3] = 256
+    _, st, _ = conv_gpu(x, w, 1, 0, (0, 255), (-255, 255), dtype=qx.I32, flags=qx.FLAG_CHECK_RANGES)
+    assert st == qx.ERR_CONTRACT
+    x[1, 3, h // 2, h // 3] = 255
+    got, st, _ = conv_gpu(x, w, 1, 0, (0, 255), (-255, 255), dtype=qx.I32, flags=qx.FLAG_CHECK_RANGES)
+    assert st == qx.OK
+    assert_exact(got, oracle.conv2d(x, w, 1, 0), "conv patches in range")
+
+
+def test_conv_explicit_patches_int16():
+    x, w = inputs.conv_case(5, 3, 21, 19, 12, 5, 5, -255, 255, seed=3)
+    got, st, info = conv_gpu(x, w, 1, 2, (-255, 255), (-255, 255))
+    assert st == qx.OK
+    assert_exact(got, oracle.conv2d(x, w, 1, 2), f"conv int16 patches {info}")
 
 
 # ------------------------------------------------ ReLU-requantize epilogue
