@@ -109,6 +109,20 @@ typedef struct {
 #define QX_FLAG_FUSED_CONVERT 8u
 #define QX_FLAG_PREPASS 16u
 
+/* Integer Conv2D plans: write the 2 x 2, stride-2 pooling of the output
+ * (after the ReLU-requantize of QX_FLAG_RELU_REQUANT when that is set)
+ * instead of the output itself -- its maximum (POOL2_MAX) or the floor of
+ * its mean (POOL2_AVG) over each window -- as NCHW (n, k_out, P / 2, Q / 2),
+ * the result of a QX_OP_MAXPOOL / QX_OP_AVGPOOL plan with r = s = stride = 2
+ * applied to the conv's output, in the conv kernel's epilogue.  The two
+ * flags exclude each other.  Requires P and Q even and a conv lowered to
+ * explicit patches whose padded image fits the packing kernel's shared
+ * memory: c < 32 and 4 (Kp + c (h + 2 pad) (w + 2 pad) + P Q) <= 49152
+ * bytes with Kp = c r s rounded up to a multiple of 8; otherwise plan
+ * creation returns QX_ERR_UNSUPPORTED. */
+#define QX_FLAG_POOL2_MAX 32u
+#define QX_FLAG_POOL2_AVG 64u
+
 typedef struct {
     qx_op op;
     qx_dtype in_dtype; /* I16 or I32 operands -> int32 output; F32 -> float */
@@ -187,8 +201,10 @@ qx_status qx_gemm_i32(qx_plan plan, const int32_t *A, const int32_t *B,
 /* GEMM-backed Conv2D (Methodology: convolution through lowering; Table 2):
  * y = conv(x, w), layouts as in qx_plan_desc.  x and w are int16, int32 or
  * float per the plan's in_dtype; y is int32 for integer plans and float for
- * F32 plans.  The lowering happens on load: no patch matrix is written to
- * device memory. */
+ * F32 plans.  With c >= 32 the lowering happens on load (im2col boxes; no
+ * patch matrix in device memory); with fewer input channels the packing
+ * kernel writes explicit FP16 patch planes into the plan's workspace.  With
+ * QX_FLAG_POOL2_MAX / _AVG, y is the pooled output (n, k_out, P/2, Q/2). */
 qx_status qx_conv2d_gemm(qx_plan plan, const void *x, const void *w, void *y,
                          qx_stream stream);
 
@@ -236,8 +252,10 @@ qx_status qx_pool2d(qx_plan plan, const void *x, void *y, qx_stream stream);
  *   -> fc 10, raw int32 logits,
  * where requant(v) = min(max(v, 0) >> shift, act_hi) is applied in the
  * producing conv / GEMM kernel's epilogue (QX_FLAG_RELU_REQUANT), so every
- * layer's operands stay inside its range contract.  Each layer is a plan of
- * this library; the executor owns the seven plans and the activations.
+ * layer's operands stay inside its range contract, and each pooling runs in
+ * the epilogue of the conv before it (QX_FLAG_POOL2_MAX / _AVG).  Each conv
+ * and fc layer is a plan of this library; the executor owns the five plans
+ * and the activations.
  * Weights (device, int32, caller-owned): w1 6x1x5x5 and w2 16x6x5x5 (KCRS),
  * w3 400x120, w4 120x84, w5 84x10 (row-major K x N, y = x w). */
 typedef struct {
@@ -251,21 +269,22 @@ typedef struct {
 
 typedef struct qx_lenet_s *qx_lenet;
 
-/* Creates the seven layer plans (setup) and one activation buffer on
+/* Creates the five layer plans (setup) and one activation buffer on
  * `device`.  Errors as qx_plan_create, e.g. CONTRACT when a layer's
  * accumulator could leave int32 under the declared ranges. */
 qx_status qx_lenet_create(const qx_lenet_desc *desc, int device, qx_lenet *out);
 
 /* logits (batch x 10 int32, device) = the pipeline on x (batch x 1 x 32 x 32
- * int32, device), asynchronous on `stream`: at most twelve kernel launches
- * (packing + tensor-core kernel per conv layer, one launch per pooling layer,
- * one or two per fc layer as its plan picks the fused or the pre-pass path). */
+ * int32, device), asynchronous on `stream`: at most ten kernel launches
+ * (packing + tensor-core kernel per conv layer, the pooling inside the
+ * latter; one or two per fc layer as its plan picks the fused or the
+ * pre-pass path). */
 qx_status qx_lenet_forward(qx_lenet net, const int32_t *x, const int32_t *w1, const int32_t *w2,
                            const int32_t *w3, const int32_t *w4, const int32_t *w5,
                            int32_t *logits, qx_stream stream);
 
 /* Synchronises the device, then returns and clears the first sticky device
- * error of the seven plans, or QX_OK. */
+ * error of the five plans, or QX_OK. */
 qx_status qx_lenet_status(qx_lenet net);
 
 /* Frees the plans and the activations.  NULL is a no-op. */

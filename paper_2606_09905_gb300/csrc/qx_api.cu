@@ -61,11 +61,14 @@ cudaError_t launch_pack_conv(bool i32, const void *x, const void *w, int n, int 
                              int k_out, int r, int s, int Cp, __half *x_planes, __half *w_planes,
                              int nx, int shift_x, int nw, int shift_w, int check, qx_range rx,
                              qx_range rw, int *err, int num_sms, cudaStream_t st);
+bool patches_image_fits(int c, int h, int w, int pad, int Kp, int64_t PQ);
 cudaError_t launch_pack_patches(bool i32, const void *x, const void *w, int n, int c, int h, int wd,
                                 int k_out, int r, int s, int stride, int pad, int P, int Q, int Kp,
                                 __half *x_planes, __half *w_planes, int nx, int shift_x, int nw,
                                 int shift_w, int check, qx_range rx, qx_range rw, int *err,
-                                int num_sms, cudaStream_t st);
+                                int pool_order, int pitch, int num_sms, cudaStream_t st);
+int patches_pitch(int c, int h, int w, int r, int s, int stride, int pad, int P, int Q, int Kp,
+                  int pool_order);
 cudaError_t attn_reassoc_prepare();
 cudaError_t attn_reassoc_launch(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_pack_attn(bool i32, const void *Q, const void *K, const void *V, int heads, int L, int d,
@@ -126,6 +129,7 @@ struct qx_plan_s {
     float *fplanes_n = nullptr, *fplanes_m = nullptr;   // FP32 kinds
     int Kp = 0, Cp = 0;
     bool conv_patches = false;                             // conv lowered to explicit patches
+    int patch_pitch = 0;                                   // staged image row pitch (0: gather kernel)
     bool fused = false;                                    // GEMM: conversion inside the kernel
     bool fused_packed = false;                             // ... on packed int16 pairs
     // attention
@@ -236,6 +240,12 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
         return fail(QX_ERR_INVALID_ARG, "QX_FLAG_FUSED_CONVERT and QX_FLAG_PREPASS apply to GEMM plans only");
     if ((d->flags & QX_FLAG_FUSED_CONVERT) && (d->flags & QX_FLAG_PREPASS))
         return fail(QX_ERR_INVALID_ARG, "QX_FLAG_FUSED_CONVERT and QX_FLAG_PREPASS exclude each other");
+    const unsigned pool2 = d->flags & (QX_FLAG_POOL2_MAX | QX_FLAG_POOL2_AVG);
+    if (pool2 && d->op != QX_OP_CONV2D)
+        return fail(QX_ERR_INVALID_ARG, "QX_FLAG_POOL2_MAX / _AVG apply to conv plans only");
+    if (pool2 == (QX_FLAG_POOL2_MAX | QX_FLAG_POOL2_AVG))
+        return fail(QX_ERR_INVALID_ARG, "QX_FLAG_POOL2_MAX and QX_FLAG_POOL2_AVG exclude each other");
+    if (pool2 && f32) return fail(QX_ERR_UNSUPPORTED, "pooled conv output is for integer plans");
     auto range_ok = [&](qx_range r) {
         if (f32) return true;   // no range contract for FP32 operands
         if (bad_range(r)) return false;
@@ -287,6 +297,16 @@ static qx_status plan_schemes(const qx_plan_desc *d, Scheme out[2], int *count, 
             }
             const int64_t Cp = (d->c + 63) / 64 * 64;
             const int64_t Kc = conv_uses_patches(d) ? (d->c * d->r * d->s + 7) / 8 * 8 : d->r * d->s * Cp;
+            if (pool2) {
+                const int64_t P = (d->h + 2 * d->pad - d->r) / d->stride + 1;
+                const int64_t Q = (d->w + 2 * d->pad - d->s) / d->stride + 1;
+                if (P % 2 != 0 || Q % 2 != 0)
+                    return fail(QX_ERR_UNSUPPORTED, "pooled conv output needs even P and Q");
+                if (!conv_uses_patches(d) || !patches_image_fits(int(d->c), int(d->h), int(d->w),
+                                                                 int(d->pad), int(Kc), P * Q))
+                    return fail(QX_ERR_UNSUPPORTED,
+                                "pooled conv output needs the staged-image patch lowering (c < 32, small image)");
+            }
             if (conv_uses_patches(d)) {
                 const int64_t P = (d->h + 2 * d->pad - d->r) / d->stride + 1;
                 const int64_t Q = (d->w + 2 * d->pad - d->s) / d->stride + 1;
@@ -695,6 +715,15 @@ static qx_status build_conv_patches(qx_plan p) {
     a.rq_shift = int(d.rq_shift);
     a.rq_hi = int(d.rq_hi);
     a.mr = mr;
+    a.pool = (d.flags & QX_FLAG_POOL2_MAX) ? 1 : (d.flags & QX_FLAG_POOL2_AVG) ? 2 : 0;
+    if (a.pool) {   // pooled output planes; the patch rows come in window order
+        a.PQ = int((P / 2) * (Q / 2));
+        a.out_row_stride = a.PQ;
+    }
+    p->patch_pitch = patches_pitch(int(d.c), int(d.h), int(d.w), int(d.r), int(d.s), int(d.stride),
+                                   int(d.pad), int(P), int(Q), p->Kp, a.pool != 0 ? 1 : 0);
+    if (a.pool && p->patch_pitch == 0)
+        return fail(QX_ERR_UNSUPPORTED, "pooled conv output needs the staged-image patch lowering");
     const int tiles = a.tiles_m * a.tiles_n;
     p->grid = std::max(1, std::min(tiles, p->num_sms));
     QX_CUDA(limb_gemm_prepare(nw, nx, mr), "kernel attributes");
@@ -1157,7 +1186,8 @@ static qx_status pack(qx_plan p, const void *a, const void *b, const void *c, cu
                                             int(d.k_out), int(d.r), int(d.s), int(d.stride),
                                             int(d.pad), P, Q, p->Kp, p->planes_m, p->planes_n,
                                             s.m.limbs, s.m.shift, s.n.limbs, s.n.shift, check,
-                                            d.range_a, d.range_b, p->err, p->num_sms, st),
+                                            d.range_a, d.range_b, p->err, p->mma.pool != 0 ? 1 : 0,
+                                            p->patch_pitch, p->num_sms, st),
                         "operand packing launch");
                 return QX_OK;
             }

@@ -1,7 +1,8 @@
 // qx_lenet.cu -- the LeNet-shaped INT32 pipeline executor (paper: Results,
 // "CNN performance": an end-to-end LeNet run on the substrate).  Host code
-// only: it chains plans of this library (two convs and three GEMMs with the
-// ReLU-requantize epilogue, two poolings) on one stream, with every
+// only: it chains plans of this library on one stream -- two convs whose
+// epilogues apply the ReLU-requantize and then the 2 x 2 pooling, three
+// GEMMs with the ReLU-requantize epilogue (none on the last) -- with every
 // activation in one device allocation made at setup.
 #include <cuda_runtime.h>
 
@@ -19,18 +20,19 @@ void set_last_error(const char *msg);   // qx_api.cu
 struct qx_lenet_s {
     qx_lenet_desc desc{};
     int device = 0;
-    qx_plan conv1 = nullptr, pool1 = nullptr, conv2 = nullptr, pool2 = nullptr;
+    qx_plan conv1 = nullptr, conv2 = nullptr;
     qx_plan fc1 = nullptr, fc2 = nullptr, fc3 = nullptr;
     void *act = nullptr;
-    int32_t *a1 = nullptr, *p1 = nullptr, *a2 = nullptr, *p2 = nullptr, *f1 = nullptr, *f2 = nullptr;
+    int32_t *p1 = nullptr, *p2 = nullptr, *f1 = nullptr, *f2 = nullptr;
 };
 
 namespace {
 
 size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
 
+// conv 5x5, stride 1, no padding, ReLU-requantize, then 2 x 2 / 2 pooling
 qx_plan_desc conv_desc(int64_t n, int64_t c, int64_t hw, int64_t k, qx_range rx, qx_range rw,
-                       int64_t shift, int64_t hi) {
+                       int64_t shift, int64_t hi, bool avg) {
     qx_plan_desc d;
     memset(&d, 0, sizeof d);
     d.op = QX_OP_CONV2D;
@@ -44,22 +46,9 @@ qx_plan_desc conv_desc(int64_t n, int64_t c, int64_t hw, int64_t k, qx_range rx,
     d.pad = 0;
     d.range_a = rx;
     d.range_b = rw;
-    d.flags = QX_FLAG_RELU_REQUANT;
+    d.flags = QX_FLAG_RELU_REQUANT | (avg ? QX_FLAG_POOL2_AVG : QX_FLAG_POOL2_MAX);
     d.rq_shift = shift;
     d.rq_hi = hi;
-    return d;
-}
-
-qx_plan_desc pool_desc(int64_t n, int64_t c, int64_t hw, bool avg) {
-    qx_plan_desc d;
-    memset(&d, 0, sizeof d);
-    d.op = avg ? QX_OP_AVGPOOL : QX_OP_MAXPOOL;
-    d.in_dtype = QX_I32;
-    d.n = n;
-    d.c = c;
-    d.h = d.w = hw;
-    d.r = d.s = 2;
-    d.stride = 2;
     return d;
 }
 
@@ -83,7 +72,7 @@ qx_plan_desc fc_desc(int64_t m, int64_t n, int64_t k, qx_range ra, qx_range rb, 
 }
 
 void destroy_plans(qx_lenet n) {
-    for (qx_plan *p : {&n->conv1, &n->pool1, &n->conv2, &n->pool2, &n->fc1, &n->fc2, &n->fc3}) {
+    for (qx_plan *p : {&n->conv1, &n->conv2, &n->fc1, &n->fc2, &n->fc3}) {
         qx_plan_destroy(*p);
         *p = nullptr;
     }
@@ -114,16 +103,15 @@ qx_status qx_lenet_create(const qx_lenet_desc *desc, int device, qx_lenet *out) 
     auto make = [&](qx_plan *p, const qx_plan_desc &d) {
         if (st == QX_OK) st = qx_plan_create(&d, device, p);
     };
-    make(&n->conv1, conv_desc(N, 1, 32, 6, desc->range_x, desc->range_w[0], desc->shift[0], desc->act_hi));
-    make(&n->pool1, pool_desc(N, 6, 28, avg));
-    make(&n->conv2, conv_desc(N, 6, 14, 16, act, desc->range_w[1], desc->shift[1], desc->act_hi));
-    make(&n->pool2, pool_desc(N, 16, 10, avg));
+    make(&n->conv1, conv_desc(N, 1, 32, 6, desc->range_x, desc->range_w[0], desc->shift[0], desc->act_hi,
+                              avg));
+    make(&n->conv2, conv_desc(N, 6, 14, 16, act, desc->range_w[1], desc->shift[1], desc->act_hi, avg));
     make(&n->fc1, fc_desc(N, 120, 400, act, desc->range_w[2], true, desc->shift[2], desc->act_hi));
     make(&n->fc2, fc_desc(N, 84, 120, act, desc->range_w[3], true, desc->shift[3], desc->act_hi));
     make(&n->fc3, fc_desc(N, 10, 84, act, desc->range_w[4], false, 0, 0));
     if (st == QX_OK) {
-        const size_t sizes[6] = {size_t(N) * 6 * 28 * 28, size_t(N) * 6 * 14 * 14, size_t(N) * 16 * 10 * 10,
-                                 size_t(N) * 400, size_t(N) * 120, size_t(N) * 84};
+        const size_t sizes[4] = {size_t(N) * 6 * 14 * 14, size_t(N) * 16 * 5 * 5, size_t(N) * 120,
+                                 size_t(N) * 84};
         size_t total = 0;
         for (size_t s : sizes) total += align256(s * 4);
         int prev = 0;
@@ -133,9 +121,9 @@ qx_status qx_lenet_create(const qx_lenet_desc *desc, int device, qx_lenet *out) 
             qx::set_last_error("LeNet activation allocation failed");
             st = QX_ERR_OOM;
         } else {
-            int32_t **slots[6] = {&n->a1, &n->p1, &n->a2, &n->p2, &n->f1, &n->f2};
+            int32_t **slots[4] = {&n->p1, &n->p2, &n->f1, &n->f2};
             char *base = static_cast<char *>(n->act);
-            for (int i = 0; i < 6; ++i) {
+            for (int i = 0; i < 4; ++i) {
                 *slots[i] = reinterpret_cast<int32_t *>(base);
                 base += align256(sizes[i] * 4);
             }
@@ -160,10 +148,8 @@ qx_status qx_lenet_forward(qx_lenet n, const int32_t *x, const int32_t *w1, cons
         return QX_ERR_INVALID_ARG;
     }
     qx_status st;
-    if ((st = qx_conv2d_gemm(n->conv1, x, w1, n->a1, stream)) != QX_OK) return st;
-    if ((st = qx_pool2d(n->pool1, n->a1, n->p1, stream)) != QX_OK) return st;
-    if ((st = qx_conv2d_gemm(n->conv2, n->p1, w2, n->a2, stream)) != QX_OK) return st;
-    if ((st = qx_pool2d(n->pool2, n->a2, n->p2, stream)) != QX_OK) return st;
+    if ((st = qx_conv2d_gemm(n->conv1, x, w1, n->p1, stream)) != QX_OK) return st;
+    if ((st = qx_conv2d_gemm(n->conv2, n->p1, w2, n->p2, stream)) != QX_OK) return st;
     if ((st = qx_gemm_i32(n->fc1, n->p2, w3, n->f1, stream)) != QX_OK) return st;
     if ((st = qx_gemm_i32(n->fc2, n->f1, w4, n->f2, stream)) != QX_OK) return st;
     return qx_gemm_i32(n->fc3, n->f2, w5, logits, stream);
@@ -172,7 +158,7 @@ qx_status qx_lenet_forward(qx_lenet n, const int32_t *x, const int32_t *w1, cons
 qx_status qx_lenet_status(qx_lenet n) {
     if (!n) return QX_ERR_INVALID_ARG;
     qx_status first = QX_OK;
-    for (qx_plan p : {n->conv1, n->pool1, n->conv2, n->pool2, n->fc1, n->fc2, n->fc3}) {
+    for (qx_plan p : {n->conv1, n->conv2, n->fc1, n->fc2, n->fc3}) {
         const qx_status st = qx_plan_status(p);
         if (first == QX_OK) first = st;
     }

@@ -260,6 +260,7 @@ struct PatchPackArgs {
     RangeCheck cx, cw;
     int *err;
     int x_blocks;          // blocks [0, x_blocks) lower x; the rest pack w
+    int pool_order;        // patch rows in 2 x 2 pooling-window order (see below)
 };
 
 // Per patch element k: the input offset of (ch, r, s) relative to the window
@@ -379,8 +380,28 @@ static InvDiv make_invdiv(int d) {
 // lower the weights exactly as pack_patches_kernel does.
 struct PatchImgArgs {
     PatchPackArgs p;
-    InvDiv by_groups, by_q, by_hwp, by_wp;
+    InvDiv by_groups, by_q, by_hwp, by_wp, by_q2;
+    int pitch;             // words per staged image row (>= w + 2 pad; picked against
+                           // shared-memory bank conflicts of the gather)
 };
+
+// Output pixel (oh, ow) of patch row `pix` of an image.  Row-major order, or
+// with pool_order the four pixels of each 2 x 2 pooling window on
+// consecutive rows, windows row-major: pix = 4 (p2 Q/2 + q2) + 2 dh + dw for
+// (oh, ow) = (2 p2 + dh, 2 q2 + dw), so that the conv kernel's epilogue finds
+// every window on four consecutive TMEM lanes.
+__device__ __forceinline__ void patch_pixel(const PatchImgArgs &pa, int pix, int &oh, int &ow) {
+    if (pa.p.pool_order) {
+        const int win = pix >> 2;
+        const int p2 = pa.by_q2.div(win);
+        const int q2 = win - p2 * (pa.p.Q >> 1);
+        oh = 2 * p2 + ((pix >> 1) & 1);
+        ow = 2 * q2 + (pix & 1);
+    } else {
+        oh = pa.by_q.div(pix);
+        ow = pix - oh * pa.p.Q;
+    }
+}
 
 template <typename T, int NX, int NW>
 __global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArgs pa) {
@@ -388,10 +409,13 @@ __global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArg
     const PatchPackArgs &p = pa.p;
     extern __shared__ int32_t psm[];
     const int Kp = p.Kp;
-    int32_t *koff = psm;                                  // Kp entries, -1 past c r s
-    int32_t *img = psm + ((Kp + 3) & ~3);
     const int hp = p.h + 2 * p.pad, wp = p.wd + 2 * p.pad;
-    const int HWp = hp * wp;
+    const int HWp = hp * wp;                              // logical padded plane
+    const int pitch = pa.pitch;
+    const int HWs = hp * pitch;                           // staged plane
+    int32_t *koff = psm;                                  // Kp entries, -1 past c r s
+    int32_t *img = psm + ((Kp + 3) & ~3);                 // c x hp x pitch, zero-padded
+    int32_t *corner = img + p.c * HWs;                    // per patch row: its window corner
     const int RSC = p.r * p.s * p.c;
     const int groups = Kp >> 3;
     if (int(blockIdx.x) >= p.x_blocks) {
@@ -422,13 +446,18 @@ __global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArg
             const int tap = k / p.c;
             const int ch = k - tap * p.c;
             const int rr = tap / p.s;
-            off = ch * HWp + rr * wp + (tap - rr * p.s);
+            off = ch * HWs + rr * pitch + (tap - rr * p.s);
         }
         koff[k] = off;
     }
     const T *X = static_cast<const T *>(p.x);
     const int HW = p.h * p.wd;
     const int PQ = p.P * p.Q;
+    for (int pix = threadIdx.x; pix < PQ; pix += blockDim.x) {   // the same for every image
+        int oh, ow;
+        patch_pixel(pa, pix, oh, ow);
+        corner[pix] = oh * p.stride * pitch + ow * p.stride;
+    }
     const int items = PQ * groups;                        // < 2^31 (the launcher checks)
     const int64_t plane_stride = int64_t(p.n) * PQ * Kp;
     const int CHWp = p.c * HWp;
@@ -437,7 +466,7 @@ __global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArg
     const int gsel = int(threadIdx.x) - pix0 * groups;    // its group of 8 elements
     const int pix_step = int(blockDim.x) / groups;
     int32_t off8[8];
-    __syncthreads();                                      // koff is complete
+    __syncthreads();                                      // both tables are complete
 #pragma unroll
     for (int e = 0; e < 8; ++e) off8[e] = fixed_g ? koff[8 * gsel + e] : -1;
     for (int im = blockIdx.x; im < p.n; im += p.x_blocks) {
@@ -448,13 +477,14 @@ __global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArg
             const int rem = i - ch * HWp;
             const int y = pa.by_wp.div(rem);
             const int iy = y - p.pad;
-            const int ix = rem - y * wp - p.pad;
+            const int xx = rem - y * wp;
+            const int ix = xx - p.pad;
             int32_t v = 0;
             if (unsigned(iy) < unsigned(p.h) && unsigned(ix) < unsigned(p.wd)) {
                 v = int32_t(xs[ch * HW + iy * p.wd + ix]);
                 p.cx.test(v, p.err);
             }
-            img[i] = v;
+            img[ch * HWs + y * pitch + xx] = v;
         }
         __syncthreads();
         __half *dst = p.x_planes + int64_t(im) * PQ * Kp;
@@ -462,12 +492,10 @@ __global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArg
             // the block is a whole number of pixels wide: this thread keeps
             // its group and its eight offsets for the whole image
             for (int pix = pix0; pix < PQ; pix += pix_step) {
-                const int oh = pa.by_q.div(pix);
-                const int ow = pix - oh * p.Q;
-                const int32_t *corner = img + oh * p.stride * wp + ow * p.stride;
+                const int32_t *cw = img + corner[pix];
                 int32_t v[8];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) v[e] = off8[e] >= 0 ? corner[off8[e]] : 0;
+                for (int e = 0; e < 8; ++e) v[e] = off8[e] >= 0 ? cw[off8[e]] : 0;
                 store_limbs8<NX>(dst + int64_t(pix) * Kp + 8 * gsel, plane_stride, v, p.shift_x);
             }
             continue;
@@ -475,14 +503,12 @@ __global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArg
         for (int it = threadIdx.x; it < items; it += blockDim.x) {
             const int pix = pa.by_groups.div(it);
             const int g = it - pix * groups;
-            const int oh = pa.by_q.div(pix);
-            const int ow = pix - oh * p.Q;
-            const int32_t *corner = img + oh * p.stride * wp + ow * p.stride;
+            const int32_t *cw = img + corner[pix];
             int32_t v[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
                 const int off = koff[8 * g + e];
-                v[e] = off >= 0 ? corner[off] : 0;
+                v[e] = off >= 0 ? cw[off] : 0;
             }
             store_limbs8<NX>(dst + int64_t(pix) * Kp + 8 * g, plane_stride, v, p.shift_x);
         }
@@ -809,6 +835,88 @@ static cudaError_t pack_patches_t(int nx, int nw, const PatchPackArgs &p, int gr
     return cudaErrorInvalidValue;
 }
 
+// Shared memory of the staged-image patch kernel: the offset table, the
+// zero-padded image (rows `pitch` words apart) and the window-corner table,
+// 32-bit words.
+static int64_t patches_image_smem(int c, int h, int pitch, int pad, int Kp, int64_t PQ) {
+    const int64_t hp = int64_t(h) + 2 * pad;
+    return (((int64_t(Kp) + 3) & ~int64_t(3)) + int64_t(c) * hp * pitch + PQ) * 4;
+}
+
+// The plan's admission test: the image fits at its narrowest pitch, w + 2 pad
+// words, and then at some pitch the launcher picks.
+bool patches_image_fits(int c, int h, int w, int pad, int Kp, int64_t PQ) {
+    return patches_image_smem(c, h, w + 2 * pad, pad, Kp, PQ) <= 48 * 1024;
+}
+
+// Threads of a staged-image block: a whole number of 8-element groups, so
+// that every thread keeps one group (and its offsets) for the whole image.
+static int patch_threads(int Kp) {
+    const int groups = Kp / 8;
+    return groups <= 256 ? groups * (256 / groups) : 256;
+}
+
+// Row pitch of the staged image: among w + 2 pad .. + 31 words (those that
+// fit), the one whose gather has the fewest shared-memory bank conflicts for
+// the first warps of an image, found by replaying the kernel's fixed-group
+// thread mapping (4 warps, every element e) on the host.  Identical words
+// are one access (broadcast); otherwise a warp access costs as many passes as
+// the most loaded of the 32 banks.
+static int pick_patch_pitch(int c, int h, int w, int r, int s, int stride, int pad, int P, int Q,
+                            int Kp, int threads, bool pool_order) {
+    // (a host search of about a million steps: the plan runs it once)
+    const int wp = w + 2 * pad, hp = h + 2 * pad;
+    const int groups = Kp / 8;
+    const int RSC = r * s * c;
+    int best = wp;
+    int64_t best_cost = -1;
+    for (int pitch = wp; pitch < wp + 32; ++pitch) {
+        if (patches_image_smem(c, h, pitch, pad, Kp, int64_t(P) * Q) > 48 * 1024) break;
+        if (threads % groups != 0) return wp;          // no fixed mapping: keep it tight
+        int64_t cost = 0;
+        for (int warp = 0; warp < 4 && warp * 32 < threads; ++warp) {
+            for (int e = 0; e < 8; ++e) {
+                int load[32] = {0};
+                int64_t seen[32];
+                int nseen = 0;
+                for (int lane = 0; lane < 32; ++lane) {
+                    const int t = warp * 32 + lane;
+                    if (t >= threads) break;
+                    const int pix = t / groups, g = t % groups;
+                    if (pix >= P * Q) continue;
+                    const int k = 8 * g + e;
+                    if (k >= RSC) continue;
+                    int oh, ow;
+                    if (pool_order) {
+                        const int win = pix >> 2;
+                        oh = 2 * (win / (Q / 2)) + ((pix >> 1) & 1);
+                        ow = 2 * (win % (Q / 2)) + (pix & 1);
+                    } else {
+                        oh = pix / Q;
+                        ow = pix % Q;
+                    }
+                    const int tap = k / c, ch = k % c, rr = tap / s, ss = tap % s;
+                    const int64_t word = int64_t(ch) * hp * pitch + int64_t(oh * stride + rr) * pitch +
+                                         (ow * stride + ss);
+                    bool dup = false;
+                    for (int i = 0; i < nseen; ++i) dup |= seen[i] == word;
+                    if (dup) continue;
+                    seen[nseen++] = word;
+                    ++load[int(word & 31)];
+                }
+                int worst = 0;
+                for (int b = 0; b < 32; ++b) worst = load[b] > worst ? load[b] : worst;
+                cost += worst;
+            }
+        }
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best = pitch;
+        }
+    }
+    return best;
+}
+
 template <typename T>
 static cudaError_t pack_patches_img_t(int nx, int nw, const PatchImgArgs &pa, int grid, int threads,
                                       int smem, cudaStream_t st) {
@@ -822,11 +930,20 @@ static cudaError_t pack_patches_img_t(int nx, int nw, const PatchImgArgs &pa, in
     return cudaErrorInvalidValue;
 }
 
+// Plan time: the staged image's row pitch, or 0 when the image does not fit
+// (the gather kernel then runs).
+int patches_pitch(int c, int h, int w, int r, int s, int stride, int pad, int P, int Q, int Kp,
+                  int pool_order) {
+    if (!patches_image_fits(c, h, w, pad, Kp, int64_t(P) * Q)) return 0;
+    if (int64_t(P) * Q * (Kp / 8) >= (int64_t(1) << 31)) return 0;
+    return pick_patch_pitch(c, h, w, r, s, stride, pad, P, Q, Kp, patch_threads(Kp), pool_order != 0);
+}
+
 cudaError_t launch_pack_patches(bool i32, const void *x, const void *w, int n, int c, int h, int wd,
                                 int k_out, int r, int s, int stride, int pad, int P, int Q, int Kp,
                                 __half *x_planes, __half *w_planes, int nx, int shift_x, int nw,
                                 int shift_w, int check, qx_range rx, qx_range rw, int *err,
-                                int num_sms, cudaStream_t st) {
+                                int pool_order, int pitch, int num_sms, cudaStream_t st) {
     PatchPackArgs p;
     p.x = x;
     p.w = w;
@@ -849,6 +966,7 @@ cudaError_t launch_pack_patches(bool i32, const void *x, const void *w, int n, i
     p.cx = make_check(check, rx);
     p.cw = make_check(check, rw);
     p.err = err;
+    p.pool_order = pool_order;
     const int64_t x_items = int64_t(n) * P * Q * (Kp / 8);
     int64_t x_blocks = (x_items + 255) / 256;
     if (x_blocks > int64_t(num_sms) * 8) x_blocks = int64_t(num_sms) * 8;
@@ -857,11 +975,12 @@ cudaError_t launch_pack_patches(bool i32, const void *x, const void *w, int n, i
     int w_blocks = int((w_items + 255) / 256);
     if (w_blocks > num_sms) w_blocks = num_sms;
     if (w_blocks < 1) w_blocks = 1;
-    // one image at a time through shared memory when it fits
+    // one image at a time through shared memory when the plan found it fits
+    // (always with pool_order, which the plan allows only then)
     const int64_t hp = int64_t(h) + 2 * pad, wp = int64_t(wd) + 2 * pad;
-    const int64_t img_words = int64_t(c) * hp * wp;
-    const int64_t smem = (((int64_t(Kp) + 3) & ~int64_t(3)) + img_words) * 4;
-    if (smem <= 48 * 1024 && int64_t(P) * Q * (Kp / 8) < (int64_t(1) << 31)) {
+    if (pitch > 0) {
+        const int threads = patch_threads(Kp);
+        const int smem = int(patches_image_smem(c, h, pitch, pad, Kp, int64_t(P) * Q));
         PatchImgArgs pa;
         pa.p = p;
         pa.p.x_blocks = n < num_sms * 8 ? n : num_sms * 8;
@@ -869,12 +988,13 @@ cudaError_t launch_pack_patches(bool i32, const void *x, const void *w, int n, i
         pa.by_q = make_invdiv(Q);
         pa.by_hwp = make_invdiv(int(hp * wp));
         pa.by_wp = make_invdiv(int(wp));
+        pa.by_q2 = make_invdiv(Q / 2 > 0 ? Q / 2 : 1);
+        pa.pitch = pitch;
         const int grid = pa.p.x_blocks + w_blocks;
-        const int groups = Kp / 8;
-        const int threads = groups <= 256 ? groups * (256 / groups) : 256;
-        return i32 ? pack_patches_img_t<int32_t>(nx, nw, pa, grid, threads, int(smem), st)
-                   : pack_patches_img_t<int16_t>(nx, nw, pa, grid, threads, int(smem), st);
+        return i32 ? pack_patches_img_t<int32_t>(nx, nw, pa, grid, threads, smem, st)
+                   : pack_patches_img_t<int16_t>(nx, nw, pa, grid, threads, smem, st);
     }
+    if (pool_order) return cudaErrorInvalidValue;
     return i32 ? pack_patches_t<int32_t>(nx, nw, p, p.x_blocks + w_blocks, st)
                : pack_patches_t<int16_t>(nx, nw, p, p.x_blocks + w_blocks, st);
 }

@@ -124,6 +124,52 @@ __device__ __forceinline__ void store_tile(const MmaArgs &a, int tm, int tn, int
     const int nrow0 = tn * T::MR + hh * T::RPT;
     const int rows = a.n_extent - nrow0;
     const int mrow = tm * kBM + q * 32 + lane;
+    if constexpr (!T::TF) {
+        if (a.pool) {
+            // 2 x 2 pooling: the four pixels of a window sit on lanes
+            // 4w .. 4w + 3 of this warp (the patch rows are in window order
+            // and the pixel count is a multiple of 4), so two butterfly
+            // shuffles combine them and lane 4w stores window w's value.
+            if (rows <= 0 || tm * kBM + q * 32 >= a.m_extent) return;   // whole warp
+            const bool lane_ok = mrow < a.m_extent;
+            const int win = mrow >> 2;
+            const int img = win / a.PQ;
+            uint32_t *o = static_cast<uint32_t *>(a.out) + int64_t(img) * a.k_out * a.PQ +
+                          (win - img * a.PQ) + int64_t(nrow0) * a.out_row_stride;
+            const bool leader = lane_ok && (lane & 3) == 0;
+            // eight rows at a time, so that their shuffles overlap
+#pragma unroll
+            for (int b = 0; b < T::RPT; b += 8) {
+                if (b >= rows) break;                  // the same for every lane
+                int32_t v[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    v[e] = int32_t(acc[b + e]);
+                    if (a.rq_on) v[e] = min(max(v[e], 0) >> a.rq_shift, a.rq_hi);
+                }
+                if (a.pool == 1) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) v[e] = max(v[e], __shfl_xor_sync(0xffffffffu, v[e], 1));
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) v[e] = max(v[e], __shfl_xor_sync(0xffffffffu, v[e], 2));
+                } else {                                 // floor of the mean, exact in 64 bits
+                    long long t[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) t[e] = v[e];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) t[e] += __shfl_xor_sync(0xffffffffu, t[e], 1);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) t[e] += __shfl_xor_sync(0xffffffffu, t[e], 2);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) v[e] = int32_t(t[e] >> 2);
+                }
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    if (leader && b + e < rows) o[int64_t(b + e) * a.out_row_stride] = uint32_t(v[e]);
+            }
+            return;
+        }
+    }
     if (rows <= 0 || mrow >= a.m_extent) return;
     int64_t lane_off = mrow;
     if (a.mode != 0) {   // conv: pixel mrow of image img, NCHW output

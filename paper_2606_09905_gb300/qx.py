@@ -27,6 +27,8 @@ FLAG_ATTN_REASSOC = 2         # attention: O = Q (K^T V), integer plans only
 FLAG_RELU_REQUANT = 4         # GEMM / conv: out = min(max(acc, 0) >> rq_shift, rq_hi)
 FLAG_FUSED_CONVERT = 8        # GEMM: one kernel converts the operands to limbs on the fly
 FLAG_PREPASS = 16             # GEMM: packing pre-pass, then the tensor-core kernel
+FLAG_POOL2_MAX = 32           # conv: write the 2x2/2 max pooling of the output
+FLAG_POOL2_AVG = 64           # conv: write the 2x2/2 floor-mean pooling of the output
 
 # Every function the header declares; the CPU tests check the exports.
 EXPORTS = ("qx_plan_create", "qx_plan_destroy", "qx_plan_query", "qx_plan_info",
@@ -264,6 +266,8 @@ class Plan:
         elif d.op == OP_CONV2D:
             P = (d.h + 2 * d.pad - d.r) // d.stride + 1
             Q = (d.w + 2 * d.pad - d.s) // d.stride + 1
+            if d.flags & (FLAG_POOL2_MAX | FLAG_POOL2_AVG):
+                P, Q = P // 2, Q // 2
             self._sx, self._sw, self._sy = S((d.n, d.c, d.h, d.w)), S((d.k_out, d.c, d.r, d.s)), S((d.n, d.k_out, P, Q))
 
     @property
@@ -398,7 +402,7 @@ LENET_WEIGHT_SHAPES = ((6, 1, 5, 5), (16, 6, 5, 5), (400, 120), (120, 84), (84, 
 
 
 class Lenet:
-    """The LeNet-shaped INT32 pipeline executor (seven plans + activations,
+    """The LeNet-shaped INT32 pipeline executor (five plans + activations,
     created once).  forward(x, weights) -> batch x 10 int32 logits."""
 
     def __init__(self, batch, range_x, ranges_w, shifts, act_hi, avg_pool=False, device=None):

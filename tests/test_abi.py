@@ -164,3 +164,28 @@ def test_gemm_path_flags_validation(lib):
     base = qx.query(qx.gemm_desc(256, 256, 256, (-1023, 1023), (-1023, 1023)))
     assert qx.query(qx.gemm_desc(256, 256, 256, (-1023, 1023), (-1023, 1023), flags=F)) == base
     assert qx.query(qx.gemm_desc(256, 256, 256, (-1023, 1023), (-1023, 1023), flags=P)) == base
+
+
+def test_pooled_conv_flags_validation(lib):
+    MX, AV = qx.FLAG_POOL2_MAX, qx.FLAG_POOL2_AVG
+    lenet1 = dict(n=8, c=1, h=32, w=32, k_out=6, r=5, s=5, stride=1, pad=0)
+
+    def conv(flags, dtype=qx.I32, **kw):
+        g = dict(lenet1, **kw)
+        return qx.conv_desc(g["n"], g["c"], g["h"], g["w"], g["k_out"], g["r"], g["s"], g["stride"],
+                            g["pad"], (0, 255), (-7, 7), dtype=dtype, flags=flags)
+
+    for f in (MX, AV):                                  # accepted on a small-channel conv
+        assert qx.query(conv(f)) == qx.query(conv(0))
+    cases = [
+        (qx.gemm_desc(8, 8, 8, (-1, 1), (-1, 1), flags=MX), qx.ERR_INVALID_ARG),   # conv only
+        (conv(MX | AV), qx.ERR_INVALID_ARG),                                       # one of the two
+        (conv(MX, dtype=qx.F32), qx.ERR_UNSUPPORTED),                              # integer plans
+        (conv(MX, h=31), qx.ERR_UNSUPPORTED),                                      # P = 27: odd
+        (conv(AV, c=64, h=16, w=16), qx.ERR_UNSUPPORTED),                          # im2col lowering
+        (conv(MX, c=16, h=64, w=64), qx.ERR_UNSUPPORTED),                          # image too large
+    ]
+    for desc, status in cases:
+        with pytest.raises(qx.QxError) as e:
+            qx.query(desc)
+        assert e.value.status == status

@@ -186,6 +186,32 @@ def test_conv_explicit_patches_int16():
     assert_exact(got, oracle.conv2d(x, w, 1, 2), f"conv int16 patches {info}")
 
 
+# --------------------------------- 2 x 2 pooling in the conv's epilogue
+@pytest.mark.parametrize("shape,stride,pad,mode,requant", [
+    ((64, 1, 32, 32, 6, 5, 5), 1, 0, "max", (4, 255)),        # LeNet conv1 + pool
+    ((64, 6, 14, 14, 16, 5, 5), 1, 0, "avg", (5, 255)),       # LeNet conv2 + pool
+    ((3, 3, 10, 12, 20, 3, 3), 1, 1, "avg", None),            # negative sums: floor
+    ((2, 4, 15, 15, 9, 3, 3), 2, 1, "max", None),
+    ((5, 2, 9, 9, 130, 2, 2), 1, 0, "max", (3, 100)),         # two N-side tiles
+])
+def test_conv_pooled_output(shape, stride, pad, mode, requant):
+    n, c, h, wd, k, r, s = shape
+    x, w = inputs.conv_case(n, c, h, wd, k, r, s, -255, 255, seed=sum(shape), dtype=torch.int32)
+    flags = qx.FLAG_POOL2_MAX if mode == "max" else qx.FLAG_POOL2_AVG
+    desc = qx.conv_desc(n, c, h, wd, k, r, s, stride, pad, (-255, 255), (-255, 255), dtype=qx.I32,
+                        flags=flags, requant=requant)
+    with qx.Plan(desc) as plan:
+        y = plan.conv2d(x.cuda(), w.cuda())
+        torch.cuda.synchronize()
+        assert plan.status() == qx.OK
+    full = oracle.conv2d(x, w, stride, pad)
+    if requant is not None:
+        full = oracle.requant(full, *requant)
+    want = oracle.pool2d(wrap32(full), 2, 2, 2, mode)
+    assert y.shape == (n, k, want.shape[2], want.shape[3])
+    assert_exact(y.cpu().numpy().astype(np.int64), want, f"pooled conv {shape} {mode} {requant}")
+
+
 # ------------------------------------------------ ReLU-requantize epilogue
 @pytest.mark.parametrize("c", [6, 64])      # explicit patches and im2col-on-load
 def test_conv_requant_epilogue(c):
