@@ -314,7 +314,11 @@ def operators(torch, qx, inputs, dev, only=None):
         r["workload"] = (f"LeNet-5-shaped INT32 pipeline, batch {batch} x 1x32x32, weights in [-7,7], "
                          f"ReLU + shift + clamp [0,255] between layers; ops = 2 x 416,520 MACs per image")
         r["images_per_s"] = round(batch / (r["execute_ms"] * 1e-3), 1)
-        nbytes = x.numel() * 4 + sum(w.numel() * 4 for w in ws) + logits.numel() * 4
+        # layer-by-layer execution: the input, the weights, and every activation
+        # between two layers written once and read once (pooled conv outputs
+        # 6x14x14 and 16x5x5, fc outputs 120 and 84), then the logits
+        act = batch * (6 * 14 * 14 + 16 * 5 * 5 + 120 + 84) * 4
+        nbytes = x.numel() * 4 + sum(w.numel() * 4 for w in ws) + 2 * act + logits.numel() * 4
         r["roofline"] = op_roofline(ops, peaks["bf16_tflops"], nbytes, peaks["hbm_gbs"], r["execute_ms"])
         return r
 
