@@ -68,6 +68,8 @@ struct MmaArgs {
     // set by the launcher from the two fields above and the kernel instance
     int k_tail_steps;         // 16-wide K sub-steps issued in the last k-block (1..4)
     int n_resident;           // one N-side tile: its k-blocks are loaded once per CTA
+    int epi_alt;              // narrow output: the two epilogue warps of a lane quarter
+                              // take alternate tiles
     int pool;                 // mode 2 only: 0, or 2 x 2 / 2 pooling of the output in the
                               // epilogue (1 max, 2 floor of the mean); the patch rows are
                               // then in pooling-window order and PQ, out_row_stride are

@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(384, 1) limb_gemm_kernel(const __grid_constant
         }
         for (int b = 0; b < T::ACC_BUFS; ++b) {
             mbar_init(&acc_full[b], 1);
-            mbar_init(&acc_empty[b], 8);
+            mbar_init(&acc_empty[b], a.epi_alt ? 4 : 8);   // the epilogue warps of one tile
         }
         mbar_init(tail, 1);
         mbar_init(n_loaded, 1);
@@ -287,10 +287,21 @@ __global__ void __launch_bounds__(384, 1) limb_gemm_kernel(const __grid_constant
     } else {
         // ------------------------------------------------------ epilogue
         const int q = warp & 3;             // TMEM lane quarter this warp may read
-        const int hh = (warp - 2) >> 2;     // which half of the N-side rows
+        const int grp = (warp - 2) >> 2;    // which of the two warps of this quarter
+        // Narrow outputs (the one N-side tile's rows all in the first half):
+        // the two warps of a quarter take alternate tiles, each on all rows,
+        // instead of one of them idling -- the per-tile epilogue is a chain
+        // of long-latency steps, and two tiles in flight per quarter overlap.
+        const int hh = a.epi_alt ? 0 : grp;                // half of the N-side rows
+        const int nchunks = (a.kblocks + a.chunk_kb - 1) / a.chunk_kb;
         uint32_t acc_it = 0;
         bool ok = true;
-        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+        int local = 0;
+        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x, ++local) {
+            if (a.epi_alt && (local & 1) != grp) {
+                acc_it += uint32_t(nchunks);                // the other warp's tile
+                continue;
+            }
             int tm, tn;
             tile_coords(t, a, tm, tn);
             // running sums: wrapping int32 (exact kind) or FP32 (TF32 kind)
@@ -365,6 +376,7 @@ static cudaError_t launch_t(const MmaArgs &a0, int grid, cudaStream_t stream) {
         if (rem > 0 && rem < kBK) a.k_tail_steps = (rem + 15) / 16;
     }
     a.n_resident = (a.tiles_n == 1 && a.kblocks >= 1 && a.kblocks <= T::STAGES) ? 1 : 0;
+    a.epi_alt = (a.tiles_n == 1 && a.n_extent <= T::RPT) ? 1 : 0;
     return launch_pdl(limb_gemm_kernel<NA, NB, KIND, MR_>, grid, T::THREADS, T::SMEM, stream, a);
 }
 
