@@ -117,9 +117,10 @@ typedef struct {
  * applied to the conv's output, in the conv kernel's epilogue.  The two
  * flags exclude each other.  Requires P and Q even and a conv lowered to
  * explicit patches whose padded image fits the packing kernel's shared
- * memory: c < 32 and 4 (Kp + c (h + 2 pad) (w + 2 pad) + P Q) <= 49152
- * bytes with Kp = c r s rounded up to a multiple of 8; otherwise plan
- * creation returns QX_ERR_UNSUPPORTED. */
+ * memory (two image buffers): c < 32 and
+ * 4 (Kp + 2 c (h + 2 pad) (w + 2 pad) + P Q) <= 49152 bytes with Kp = c r s
+ * rounded up to a multiple of 8; otherwise plan creation returns
+ * QX_ERR_UNSUPPORTED. */
 #define QX_FLAG_POOL2_MAX 32u
 #define QX_FLAG_POOL2_AVG 64u
 

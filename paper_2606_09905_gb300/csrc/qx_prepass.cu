@@ -413,9 +413,10 @@ __global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArg
     const int HWp = hp * wp;                              // logical padded plane
     const int pitch = pa.pitch;
     const int HWs = hp * pitch;                           // staged plane
+    const int IMG = p.c * HWs;                            // words of one staged image
     int32_t *koff = psm;                                  // Kp entries, -1 past c r s
-    int32_t *img = psm + ((Kp + 3) & ~3);                 // c x hp x pitch, zero-padded
-    int32_t *corner = img + p.c * HWs;                    // per patch row: its window corner
+    int32_t *img = psm + ((Kp + 3) & ~3);                 // 2 x c x hp x pitch, zero-padded
+    int32_t *corner = img + 2 * IMG;                      // per patch row: its window corner
     const int RSC = p.r * p.s * p.c;
     const int groups = Kp >> 3;
     if (int(blockIdx.x) >= p.x_blocks) {
@@ -469,8 +470,11 @@ __global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArg
     __syncthreads();                                      // both tables are complete
 #pragma unroll
     for (int e = 0; e < 8; ++e) off8[e] = fixed_g ? koff[8 * gsel + e] : -1;
-    for (int im = blockIdx.x; im < p.n; im += p.x_blocks) {
-        __syncthreads();                                  // the previous image is consumed
+    // Stage image `im` into buffer `buf`: 32-bit inputs by asynchronous
+    // copies (one commit group per image, so the next image's loads overlap
+    // this image's gather), 16-bit ones by plain loads.  Padding is zeroed.
+    auto stage = [&](int im, int buf) {
+        int32_t *dimg = img + buf * IMG;
         const T *xs = X + int64_t(im) * p.c * HW;
         for (int i = threadIdx.x; i < CHWp; i += blockDim.x) {
             const int ch = pa.by_hwp.div(i);
@@ -479,39 +483,69 @@ __global__ void __launch_bounds__(256) pack_patches_img_kernel(const PatchImgArg
             const int iy = y - p.pad;
             const int xx = rem - y * wp;
             const int ix = xx - p.pad;
-            int32_t v = 0;
+            int32_t *d = dimg + ch * HWs + y * pitch + xx;
             if (unsigned(iy) < unsigned(p.h) && unsigned(ix) < unsigned(p.wd)) {
-                v = int32_t(xs[ch * HW + iy * p.wd + ix]);
-                p.cx.test(v, p.err);
+                const T *src = xs + ch * HW + iy * p.wd + ix;
+                if constexpr (sizeof(T) == 4) {
+                    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(d)), "l"(src)
+                                 : "memory");
+                } else {
+                    *d = int32_t(*src);
+                }
+            } else {
+                *d = 0;
             }
-            img[ch * HWs + y * pitch + xx] = v;
         }
-        __syncthreads();
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    int buf = 0;
+    if (int(blockIdx.x) < p.n) stage(blockIdx.x, 0);
+    for (int im = blockIdx.x; im < p.n; im += p.x_blocks, buf ^= 1) {
+        const int next = im + p.x_blocks;
+        if (next < p.n) {
+            stage(next, buf ^ 1);                         // read by nobody since the last barrier
+            asm volatile("cp.async.wait_group 1;" ::: "memory");
+        } else {
+            asm volatile("cp.async.wait_group 0;" ::: "memory");
+        }
+        __syncthreads();                                  // image `im` is staged
+        const int32_t *cimg = img + buf * IMG;
+        if (p.cx.on) {                                    // the range contract, once per value
+            for (int i = threadIdx.x; i < CHWp; i += blockDim.x) {
+                const int ch = pa.by_hwp.div(i);
+                const int rem = i - ch * HWp;
+                const int y = pa.by_wp.div(rem);
+                const int xx = rem - y * wp;
+                if (unsigned(y - p.pad) < unsigned(p.h) && unsigned(xx - p.pad) < unsigned(p.wd))
+                    p.cx.test(cimg[ch * HWs + y * pitch + xx], p.err);
+            }
+        }
         __half *dst = p.x_planes + int64_t(im) * PQ * Kp;
         if (fixed_g) {
             // the block is a whole number of pixels wide: this thread keeps
             // its group and its eight offsets for the whole image
             for (int pix = pix0; pix < PQ; pix += pix_step) {
-                const int32_t *cw = img + corner[pix];
+                const int32_t *cw = cimg + corner[pix];
                 int32_t v[8];
 #pragma unroll
                 for (int e = 0; e < 8; ++e) v[e] = off8[e] >= 0 ? cw[off8[e]] : 0;
                 store_limbs8<NX>(dst + int64_t(pix) * Kp + 8 * gsel, plane_stride, v, p.shift_x);
             }
-            continue;
-        }
-        for (int it = threadIdx.x; it < items; it += blockDim.x) {
-            const int pix = pa.by_groups.div(it);
-            const int g = it - pix * groups;
-            const int32_t *cw = img + corner[pix];
-            int32_t v[8];
+        } else {
+            for (int it = threadIdx.x; it < items; it += blockDim.x) {
+                const int pix = pa.by_groups.div(it);
+                const int g = it - pix * groups;
+                const int32_t *cw = cimg + corner[pix];
+                int32_t v[8];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                const int off = koff[8 * g + e];
-                v[e] = off >= 0 ? cw[off] : 0;
+                for (int e = 0; e < 8; ++e) {
+                    const int off = koff[8 * g + e];
+                    v[e] = off >= 0 ? cw[off] : 0;
+                }
+                store_limbs8<NX>(dst + int64_t(pix) * Kp + 8 * g, plane_stride, v, p.shift_x);
             }
-            store_limbs8<NX>(dst + int64_t(pix) * Kp + 8 * g, plane_stride, v, p.shift_x);
         }
+        __syncthreads();                                  // buffer `buf` is free again
     }
 }
 
@@ -835,12 +869,12 @@ static cudaError_t pack_patches_t(int nx, int nw, const PatchPackArgs &p, int gr
     return cudaErrorInvalidValue;
 }
 
-// Shared memory of the staged-image patch kernel: the offset table, the
-// zero-padded image (rows `pitch` words apart) and the window-corner table,
-// 32-bit words.
+// Shared memory of the staged-image patch kernel: the offset table, two
+// zero-padded image buffers (rows `pitch` words apart) and the window-corner
+// table, 32-bit words.
 static int64_t patches_image_smem(int c, int h, int pitch, int pad, int Kp, int64_t PQ) {
     const int64_t hp = int64_t(h) + 2 * pad;
-    return (((int64_t(Kp) + 3) & ~int64_t(3)) + int64_t(c) * hp * pitch + PQ) * 4;
+    return (((int64_t(Kp) + 3) & ~int64_t(3)) + 2 * int64_t(c) * hp * pitch + PQ) * 4;
 }
 
 // The plan's admission test: the image fits at its narrowest pitch, w + 2 pad
