@@ -229,3 +229,25 @@ def test_int8_mma_peak_measurement():
     tops = qx.measure_int8_mma_peak(0)
     assert 1.0 < tops < 1e5
     assert qx.load().qx_measure_int8_mma_peak(0, None) == qx.ERR_INVALID_ARG
+
+
+# Narrow outputs exercise the short-tile paths of the limb kernel: the N side
+# (rows of C) in one tile loaded once per CTA when its k-blocks fit the stage
+# ring, the last k-block's empty K sub-steps skipped, and the two epilogue
+# warps of a lane quarter taking alternate tiles when every row of C falls in
+# the first half of the tile -- with one FP32 chunk per tile or several.
+@pytest.mark.parametrize("M,N,K,lim,dtype", [
+    (6, 1000, 40, 255, torch.int16),        # resident N side, 3 of 4 sub-steps, one chunk
+    (8, 4096, 100, 1023, torch.int16),      # 2 k-blocks, tail of 3 sub-steps
+    (20, 777, 5000, 2000, torch.int32),     # many chunks, N side re-loaded per tile
+    (40, 300, 130, 255, torch.int32),       # rows past the first half: no alternation
+    (33, 2000, 17, 7, torch.int32),         # one sub-step of one k-block
+])
+def test_narrow_outputs(M, N, K, lim, dtype):
+    A, B, ref, _ = _case(M, N, K, -lim, lim, seed=M * 7 + K, dtype=dtype)
+    dt = qx.I16 if dtype == torch.int16 else qx.I32
+    got, st, info = gemm_gpu(A, B, (-lim, lim), (-lim, lim), dtype=dt, path="prepass")
+    assert st == qx.OK
+    if (M, N, K) == (20, 777, 5000):
+        assert info[0]["n_chunks"] > 1
+    assert_exact(got, wrap32(ref), f"narrow GEMM {M}x{N}x{K} {info}")
