@@ -602,8 +602,13 @@ def run_qx(args):
     peak = peaks["bf16_tflops_sustained"] if long_run else peaks["bf16_tflops"]
     peak_kind = "sustained" if long_run else "burst"
     pack_bytes = (M * K + K * N) * 2 + (scheme["limbs_a"] * M * K + scheme["limbs_b"] * N * K) * 2
+    # DRAM bytes of one launch of this kernel at 8192^3 (dram__bytes_read.sum +
+    # dram__bytes_write.sum, one single-pass ncu capture of the current kernel,
+    # profiles/limb_gemm_8192_dram.md); other sizes have no capture
+    traffic = 1.98e9 + 258.08e6 if (M, N, K) == (8192, 8192, 8192) else None
     roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
-                "frac": round(achieved / peak, 4), "traffic": None,
+                "frac": round(achieved / peak, 4), "traffic": traffic,
+                "algorithmic_bytes": (scheme["limbs_a"] * M * K + scheme["limbs_b"] * N * K) * 2 + M * N * 4,
                 "kernel": "qx::limb_gemm_kernel<2,1>", "kernel_ms": round(kernel_ms, 4),
                 "peak_source": f"{peaks['source']} dense bf16 {peak_kind} (FP16 runs at the BF16 rate); "
                                f"timed loop {ms_total / 1e3:.2f} s",
