@@ -31,6 +31,7 @@ void scheme_to_info(const Scheme &s, qx_scheme_info *o);
 bool limb_gemm_supported(int na, int nb);
 int limb_gemm_rows_per_limb(int na);
 int limb_gemm_pick_rows(int na, int64_t m_extent, int64_t n_extent, int num_sms);
+int limb_gemm_pick_rows_conv(int na, int64_t m_extent, int64_t n_extent, int num_sms);
 cudaError_t limb_gemm_prepare(int na, int nb, int mr);
 cudaError_t limb_gemm_launch(int na, int nb, const MmaArgs &a, int grid, cudaStream_t stream);
 bool fused_gemm_packed_ok(int na, int shift_n, int nb, int shift_m, bool values_fit_int16);
@@ -738,7 +739,7 @@ static qx_status build_conv(qx_plan p) {
     const int nw = s.n.limbs, nx = s.m.limbs;
     const int64_t P = (d.h + 2 * d.pad - d.r) / d.stride + 1;
     const int64_t Q = (d.w + 2 * d.pad - d.s) / d.stride + 1;
-    const int mr = limb_gemm_pick_rows(nw, d.n * P * Q, d.k_out, p->num_sms);
+    const int mr = limb_gemm_pick_rows_conv(nw, d.n * P * Q, d.k_out, p->num_sms);
     p->Cp = int((d.c + 63) / 64 * 64);
     const size_t x_bytes = size_t(nx) * d.n * d.h * d.w * p->Cp * 2;
     const size_t w_bytes = size_t(nw) * d.k_out * d.r * d.s * p->Cp * 2;

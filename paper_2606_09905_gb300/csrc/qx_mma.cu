@@ -430,6 +430,19 @@ int limb_gemm_pick_rows(int na, int64_t m_extent, int64_t n_extent, int num_sms)
     return 0.6 * double(r_half) < double(r_full) ? 64 : mr;
 }
 
+// Tile height for a conv lowered on load (im2col M side).  With one weight
+// digit a 64-row tile's MMAs have N = 64 and run at half rate, so a half
+// tile costs about as much as a full one: halve only when that takes fewer
+// rounds of tiles (Table 2 conv: 196 full tiles are two rounds, 392 half
+// tiles three, 15.8 -> 14.4 us with full tiles).  Otherwise as for GEMMs.
+int limb_gemm_pick_rows_conv(int na, int64_t m_extent, int64_t n_extent, int num_sms) {
+    if (na != 1 || num_sms < 1) return limb_gemm_pick_rows(na, m_extent, n_extent, num_sms);
+    const int64_t tm = (m_extent + kBM - 1) / kBM;
+    const int64_t r_full = (tm * ((n_extent + 127) / 128) + num_sms - 1) / num_sms;
+    const int64_t r_half = (tm * ((n_extent + 63) / 64) + num_sms - 1) / num_sms;
+    return r_half < r_full ? 64 : 128;
+}
+
 cudaError_t limb_gemm_prepare(int na, int nb, int mr) { QX_LIMB_DISPATCH(prepare_t) }
 
 cudaError_t limb_gemm_launch(int na, int nb, const MmaArgs &a, int grid, cudaStream_t stream) {
