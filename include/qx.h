@@ -109,7 +109,8 @@ typedef struct {
 #define QX_FLAG_FUSED_CONVERT 8u
 #define QX_FLAG_PREPASS 16u
 
-/* Integer Conv2D plans: write the 2 x 2, stride-2 pooling of the output
+/* Integer Conv2D plans (the pooling rows of Table 2 fused into the conv of
+ * the Results' LeNet run): write the 2 x 2, stride-2 pooling of the output
  * (after the ReLU-requantize of QX_FLAG_RELU_REQUANT when that is set)
  * instead of the output itself -- its maximum (POOL2_MAX) or the floor of
  * its mean (POOL2_AVG) over each window -- as NCHW (n, k_out, P / 2, Q / 2),
