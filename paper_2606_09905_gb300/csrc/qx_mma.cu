@@ -20,12 +20,16 @@
 //
 // Roles (one CTA per SM, persistent over output tiles):
 //   warps 0, 11 M-side TMA producers (one thread each, alternate k-blocks)
-//   warp 10     N-side TMA producer: stage ring of `STAGES` buffers
+//   warp 10     N-side TMA producer: stage ring of `STAGES` buffers, or, when
+//               the N side is one tile that fits the ring, all of it once
 //   warp 1      TMEM owner and MMA issuer (one thread)
 //   warps 2..9  epilogue: two warps per TMEM lane quarter, each owning half
-//               of the N-side rows; running int32 sums live in registers.
-// Accumulators are double-buffered in TMEM whenever they fit in 256 columns,
-// so the epilogue drains chunk c while the tensor cores run chunk c + 1.
+//               of the N-side rows (or, for narrow outputs, alternate tiles);
+//               running int32 sums live in registers.
+// Accumulators are double-buffered in TMEM whenever they fit in 256 columns
+// and quadruple-buffered within 128, so the epilogue drains chunk c while
+// the tensor cores run the chunks after it.  Conv mode 2 can pool 2 x 2
+// windows in the epilogue (see store_tile).
 //
 // FP32 kind (Table 2 FP32 conv row).  The same pipeline runs kind::tf32 with
 // FP32 operands split as x = x_big + x_small (both TF32-rounded): each k-step
