@@ -6,9 +6,12 @@
 // every element (an exact FP16 integer), laid out K-major so the TMA loads of
 // the tiled limb GEMM read 128-byte rows.  The GEMM's B is transposed on the
 // way (K x N -> N x K); the conv input goes NCHW -> NHWC with channels padded
-// to a multiple of 64 (zeros); conv weights go KCRS -> K,R,S,C.  With range
-// checking on, every operand is compared with its declared range and a
-// violation sets QX_ERR_CONTRACT in the plan's device error word.
+// to a multiple of 64 (zeros); conv weights go KCRS -> K,R,S,C.  Convs with
+// fewer than 32 input channels get explicit patch planes instead (one row per
+// output pixel, k = (r S + s) C + c), built one staged image at a time, in
+// pooling-window order when the conv's epilogue pools.  With range checking
+// on, every operand is compared with its declared range and a violation sets
+// QX_ERR_CONTRACT in the plan's device error word.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
