@@ -435,8 +435,8 @@ def run_reference(args):
     if rank != 0:
         return 0
     steps, warmup = args.steps, args.warmup
-    # size each step so warm-up + timed steps take about two minutes in all
-    per_step_s = max(0.5, 120.0 / max(1, steps + warmup))
+    # size each step so warm-up + timed steps take about --ref-seconds in all
+    per_step_s = max(0.05, args.ref_seconds / max(1, steps + warmup))
     rows = calibrate_rows(per_step_s)
     for _ in range(warmup):
         cpu_oracle_gemm(rows)
@@ -677,6 +677,8 @@ def main():
     ap.add_argument("--no-operators", action="store_true", help="skip the conv/attention timings")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--ref-seconds", type=float, default=120.0,
+                    help="reference arm: CPU time for warm-up + timed steps together")
     ap.add_argument("--size", type=int, default=8192,
                     help="M = N = K of the GEMM step (8192 is the benchmark workload; smaller "
                          "sizes exist for profiling captures)")
