@@ -189,3 +189,22 @@ def test_pooled_conv_flags_validation(lib):
         with pytest.raises(qx.QxError) as e:
             qx.query(desc)
         assert e.value.status == status
+
+
+def test_pooled_conv_shared_memory_limit(lib):
+    """The documented admission rule: 4 (Kp + 2 c (h + 2 pad)(w + 2 pad) + P Q)
+    <= 49152 bytes.  c = 1, 3x3, pad 0: Kp = 16; h = w = 64 needs
+    4 (16 + 8192 + 3844) = 48208 bytes (accepted), h = w = 66 needs
+    4 (16 + 8712 + 4096) = 51296 (refused)."""
+    def desc(hw):
+        return qx.conv_desc(2, 1, hw, hw, 8, 3, 3, 1, 0, (0, 255), (-7, 7), dtype=qx.I32,
+                            flags=qx.FLAG_POOL2_MAX)
+    for hw, ok in ((64, True), (66, False)):
+        words = 16 + 2 * hw * hw + (hw - 2) ** 2
+        assert (4 * words <= 49152) == ok
+        if ok:
+            assert len(qx.query(desc(hw))) == 1
+        else:
+            with pytest.raises(qx.QxError) as e:
+                qx.query(desc(hw))
+            assert e.value.status == qx.ERR_UNSUPPORTED
