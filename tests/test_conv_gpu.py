@@ -193,6 +193,7 @@ def test_conv_explicit_patches_int16():
     ((3, 3, 10, 12, 20, 3, 3), 1, 1, "avg", None),            # negative sums: floor
     ((2, 4, 15, 15, 9, 3, 3), 2, 1, "max", None),
     ((5, 2, 9, 9, 130, 2, 2), 1, 0, "max", (3, 100)),         # two N-side tiles
+    ((2, 1, 64, 64, 8, 3, 3), 1, 0, "avg", (2, 255)),         # largest staged image (48208 B)
 ])
 def test_conv_pooled_output(shape, stride, pad, mode, requant):
     n, c, h, wd, k, r, s = shape
