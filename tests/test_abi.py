@@ -208,3 +208,26 @@ def test_pooled_conv_shared_memory_limit(lib):
             with pytest.raises(qx.QxError) as e:
                 qx.query(desc(hw))
             assert e.value.status == qx.ERR_UNSUPPORTED
+
+
+def test_noalloc_argument_checks_run_before_any_device_work(lib):
+    """The allocation-free GEMM refuses bad arguments on the host; the fake
+    (never dereferenced) pointers below are only tested for null and
+    alignment."""
+    R = qx.Range
+    A, B, C = ctypes.c_void_p(0x10000), ctypes.c_void_p(0x20000), ctypes.c_void_p(0x30000)
+    f = lib.qx_gemm_i16_i32_noalloc
+    ok_r = R(-1023, 1023)
+    assert f(-1, 8, 8, ok_r, ok_r, 0, A, B, C, None, None) == qx.ERR_INVALID_ARG
+    assert f(8, 8, 8, R(5, 1), ok_r, 0, A, B, C, None, None) == qx.ERR_INVALID_ARG        # empty
+    assert f(8, 8, 8, ok_r, R(-40000, 1), 0, A, B, C, None, None) == qx.ERR_INVALID_ARG  # not int16
+    assert f(0, 8, 8, ok_r, ok_r, 0, None, None, None, None, None) == qx.OK              # nothing to do
+    assert f(8, 8, 8, ok_r, ok_r, 0, A, B, None, None, None) == qx.ERR_INVALID_ARG       # null C
+    assert f(8, 8, 8, ok_r, ok_r, 0, ctypes.c_void_p(0x10008), B, C, None, None) == qx.ERR_UNSUPPORTED
+    # limb planes beyond the static scratch, and K not a multiple of 8 for the fused path
+    assert f(4096, 4096, 4001, ok_r, ok_r, 0, A, B, C, None, None) == qx.ERR_UNSUPPORTED
+    assert b"scratch" in lib.qx_last_error()
+
+
+def test_int8_peak_measurement_rejects_null_output(lib):
+    assert lib.qx_measure_int8_mma_peak(0, None) == qx.ERR_INVALID_ARG
