@@ -350,3 +350,63 @@ def test_lenet_pass_through_network():
     m = m.reshape(3, 5, 2, 5, 2).max(axis=(2, 4))           # pool2
     want = m.reshape(3, -1).sum(axis=1)
     assert logits.shape == (3, 10) and (logits == want[:, None]).all()
+
+
+# ------------------------------------------ seeded random sweeps (CPU only)
+# Many small random shapes against the independent routines above: torch
+# float64 conv2d and pooling (exact for these integer magnitudes, far below
+# 2^53) and numpy int64 matmul, so that an index or padding slip that only
+# shows at particular sizes, strides or paddings fails somewhere.
+@pytest.mark.parametrize("seed", range(4))
+def test_conv_random_shapes_match_torch(seed):
+    rng = np.random.default_rng(500 + seed)
+    for _ in range(8):
+        n, c, k = (int(v) for v in rng.integers(1, 4, size=3))
+        r, s = (int(v) for v in rng.integers(1, 6, size=2))
+        stride = int(rng.integers(1, 4))
+        pad = int(rng.integers(0, 3))
+        h = int(rng.integers(max(1, r - 2 * pad), 13))
+        w = int(rng.integers(max(1, s - 2 * pad), 13))
+        x = torch.from_numpy(rng.integers(-255, 256, size=(n, c, h, w)))
+        wt = torch.from_numpy(rng.integers(-255, 256, size=(k, c, r, s)))
+        ref = torch.nn.functional.conv2d(x.double(), wt.double(), stride=stride, padding=pad)
+        got = oracle.conv2d(x.numpy(), wt.numpy(), stride, pad)
+        assert got.shape == tuple(ref.shape), (n, c, h, w, k, r, s, stride, pad)
+        assert (got == ref.numpy().astype(np.int64)).all(), (n, c, h, w, k, r, s, stride, pad)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_gemm_random_shapes_match_numpy(seed):
+    rng = np.random.default_rng(600 + seed)
+    for _ in range(10):
+        M, N, K = (int(v) for v in rng.integers(1, 40, size=3))
+        A = rng.integers(-32768, 32768, size=(M, K))
+        B = rng.integers(-32768, 32768, size=(K, N))
+        C, _ = oracle.gemm(A, B)
+        assert (C == A @ B).all(), (M, N, K)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_pool_random_shapes_match_torch(seed):
+    rng = np.random.default_rng(700 + seed)
+    for _ in range(8):
+        k = int(rng.integers(1, 4))
+        s = int(rng.integers(1, 4))
+        n, c = (int(v) for v in rng.integers(1, 3, size=2))
+        h, w = (int(v) for v in rng.integers(k, 11, size=2))
+        x = rng.integers(-10**6, 10**6, size=(n, c, h, w))
+        xt = torch.from_numpy(x.astype(np.float64))
+        assert (oracle.pool2d(x, k, k, s, "max") == torch.nn.functional.max_pool2d(xt, k, s).numpy()).all()
+        sums = np.rint(torch.nn.functional.avg_pool2d(xt, k, s).numpy() * (k * k)).astype(np.int64)
+        assert (oracle.pool2d(x, k, k, s, "avg") == np.floor_divide(sums, k * k)).all()
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_attention_random_shapes_match_numpy(seed):
+    rng = np.random.default_rng(800 + seed)
+    for _ in range(6):
+        L, d = int(rng.integers(1, 70)), int(rng.integers(1, 40))
+        Q, K, V = (rng.integers(-7, 8, size=(L, d)) for _ in range(3))
+        O = oracle.attn(Q, K, V)
+        O = O[0] if isinstance(O, tuple) else O
+        assert (np.asarray(O) == (Q @ K.T) @ V).all(), (L, d)
