@@ -226,3 +226,41 @@ def test_conv_requant_epilogue(c):
     want = oracle.requant(oracle.conv2d(x, w, 1, 1), 9, 1000)
     assert 0 < (want == 1000).sum() < want.size and (want == 0).any()   # both clamps exercised
     assert_exact(y.cpu().numpy().astype(np.int64), want, f"conv requant c={c}")
+
+
+# ----------------------------------------------- seeded random shape sweep
+@pytest.mark.parametrize("seed", range(3))
+def test_conv_random_shapes(seed):
+    """Random shapes through both lowerings (explicit patches below 32 input
+    channels, im2col on load above), int16 and int32, with the pooled epilogue
+    whenever P and Q come out even on the patch path; bit-exact against the
+    oracle."""
+    rng = np.random.default_rng(900 + seed)
+    for _ in range(6):
+        c = int(rng.choice([1, 2, 5, 17, 31, 40, 70]))
+        n, k = int(rng.integers(1, 4)), int(rng.integers(1, 70))
+        r, s = (int(v) for v in rng.integers(1, 6, size=2))
+        stride, pad = int(rng.integers(1, 4)), int(rng.integers(0, 3))
+        h = int(rng.integers(max(1, r - 2 * pad), 21))
+        w = int(rng.integers(max(1, s - 2 * pad), 21))
+        dt = torch.int16 if rng.integers(0, 2) else torch.int32
+        lim = 255
+        x, wt = inputs.conv_case(n, c, h, w, k, r, s, -lim, lim, seed=int(rng.integers(1 << 30)), dtype=dt)
+        qdt = qx.I16 if dt == torch.int16 else qx.I32
+        full = oracle.conv2d(x, wt, stride, pad)
+        P, Q = full.shape[2], full.shape[3]
+        pool = c < 32 and P % 2 == 0 and Q % 2 == 0 and rng.integers(0, 2) == 1
+        flags = qx.FLAG_POOL2_MAX if pool else 0
+        try:
+            plan = qx.Plan(qx.conv_desc(n, c, h, w, k, r, s, stride, pad, (-lim, lim), (-lim, lim),
+                                        dtype=qdt, flags=flags))
+        except qx.QxError as e:
+            assert pool and e.status == qx.ERR_UNSUPPORTED     # image too large to stage
+            continue
+        with plan:
+            y = plan.conv2d(x.cuda(), wt.cuda())
+            torch.cuda.synchronize()
+            assert plan.status() == qx.OK
+        want = oracle.pool2d(full, 2, 2, 2, "max") if pool else full
+        assert_exact(y.cpu().numpy().astype(np.int64), want,
+                     f"conv n{n} c{c} {h}x{w} k{k} {r}x{s} s{stride} p{pad} {dt} pool={pool}")
